@@ -1,0 +1,141 @@
+/*
+ * codecgauge.h -- C ABI of libcodecgauge, the GB300 (sm_103a) encode/decode path of
+ * Codec-Gauge's inference-time cache-coordinate layer (arxiv 2607.20538).
+ *
+ * The method (Sec. 3, the encode/decode equations): for every layer l, cache type
+ * s in {K, V}, head h and channel group r, a fixed orthogonal gauge G_{l,s,h,r}
+ * (g x g) maps each g-channel slice of a cached key/value vector into codec-facing
+ * coordinates, Z = G X; a fixed backend codes Z into a byte buffer B_c = C(Z); decode
+ * recovers Zhat = D(B_c) and restores Xhat = G^{-1} Zhat = G^T Zhat (Sec. 4.1: the
+ * gauge is exp(A - A^T), so its inverse is its transpose). The gauge mixes channels
+ * only inside a group; it never mixes tokens, heads or layers (Sec. 1, Sec. 3).
+ * Backends (Sec. 4.3): block-uniform asymmetric min/max quantization and KIVI-style
+ * quantization (per-channel key ranges, per-token value ranges, full-precision
+ * residual window), at 2, 3, 4, 6 or 8 bits.
+ *
+ * Conventions shared by every entry point
+ *   - All data pointers are DEVICE pointers owned by the caller. The library never
+ *     allocates, frees or retains them. Calls are asynchronous on `stream`
+ *     (a cudaStream_t passed as void*; NULL = legacy default stream).
+ *   - Every entry point returns an int status: CG_OK or a negative CG_E* code. On a
+ *     negative status nothing was launched; cg_last_error() returns a message.
+ *   - Numbers: bf16 = IEEE binary16-brain (8-bit significand), fp16 = IEEE binary16,
+ *     fp32 = IEEE binary32, all little-endian.
+ *
+ * Tensor layouts (row-major, leftmost index slowest; layer-major so one layer's bytes
+ * are contiguous and a per-layer call is made with L = 1 and pointers offset by the
+ * L = 1 byte counts of cg_packed_bytes):
+ *   KV input/output  X  : bf16 [L][2][B][H][T][d]      (s = 0 keys, s = 1 values; Sec. 3)
+ *   gauges           G  : fp32 [L][2][H][d/g][g][g]    G[i][j] row-major, z_i = sum_j G[i][j] x_j
+ *   block-uniform (CG_BLOCK_UNIFORM), history of T_cap tokens:
+ *     codes  : u8    [L][2][B][H][T_cap][d/block][block*bits/8]
+ *     scales : half2 [L][2][B][H][T_cap][d/block]      .x = scale s, .y = zero (block min m)
+ *   KIVI-style (CG_KIVI), n_q = max(0, floor((T - residual)/block)) * block quantized tokens:
+ *     codes  per layer: keys  u8 [B][H][n_q/block][d][block*bits/8]   (per-channel token streams)
+ *                       then values u8 [B][H][n_q][d/block][block*bits/8]
+ *     scales per layer: keys  half2 [B][H][n_q/block][d], then values half2 [B][H][n_q][d/block]
+ *     residual        : bf16 [L][2][B][H][T - n_q][d]   newest tokens, raw (un-gauged) X
+ *   no-compression (CG_NONE, the sanity rows of Sec. 4.4):
+ *     codes  : fp32 [L][2][B][H][T_cap][d]  the gauge-space tensor Z itself
+ *
+ * Bit packing: inside one block payload, code k occupies bits [k*bits, (k+1)*bits) of a
+ * little-endian bit stream (bit 0 = LSB of byte 0). For KIVI keys a "block" is the
+ * stream of `block` consecutive tokens of one channel.
+ *
+ * Quantization rule (Sec. 4.3 names an asymmetric min/max range per block; the
+ * arithmetic below is this library's fixed reading of it):
+ *   z      = fp32 gauge-space value; each z_i is the left-to-right fp32 fused
+ *            multiply-add chain acc = fma(G[i][j], x_j, acc), j = 0..g-1, acc0 = +0.
+ *   s32    = (max - min) / (2^bits - 1) over the block (fp32 subtract, fp32 divide)
+ *   s, m   = fp16 round-to-nearest-even of s32 and of min; stored as half2 {s, m}
+ *   q      = clamp(rint((z - m) / s), 0, 2^bits - 1)  (fp32; q = 0 when s == 0)
+ *   decode : zhat = q * s + m ; xhat_i = sum_j G[j][i] zhat_j ; bf16 round-to-nearest-even.
+ */
+#ifndef CODECGAUGE_H
+#define CODECGAUGE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define CG_OK            0
+#define CG_EINVAL       (-1)  /* a bad argument: shape, parameter, null or misaligned pointer  */
+#define CG_EUNSUPPORTED (-2)  /* valid in the method but not provided (e.g. KIVI append)        */
+#define CG_ECUDA        (-3)  /* a CUDA launch or runtime call failed; see cg_last_error()      */
+#define CG_ERANGE       (-4)  /* a byte count or index does not fit the library's integer types */
+
+/* Backends (Sec. 4.3 compression conditions; CG_NONE = the no-compression rows of Sec. 4.4). */
+#define CG_BLOCK_UNIFORM 0
+#define CG_KIVI          1
+#define CG_NONE          2
+
+/* Device status bits, accumulated by kernels and read by cg_get_status(). */
+#define CG_FLAG_NONFINITE_INPUT 0x1  /* a NaN/Inf bf16 input value was seen                 */
+#define CG_FLAG_FP16_OVERFLOW   0x2  /* a block scale or zero did not fit in fp16 (became inf) */
+#define CG_FLAG_PIPE_TIMEOUT    0x4  /* a bounded pipeline wait gave up; outputs are invalid  */
+
+/* Cache shape (Sec. 3 notation: B batch, H KV heads, T tokens, d head dimension, L layers).
+ * d in {32, 64, 128, 256}; L*2*H <= 65535 and L*B*H <= 65535.
+ * t0, T_cap: block-uniform only. Encode writes tokens [t0, t0+T) of a history that holds
+ * T_cap tokens per (l, s, b, h); decode reads tokens [t0, t0+T) of it and writes a dense
+ * [L][2][B][H][T][d] output. T_cap = 0 means T_cap = t0 + T. KIVI requires t0 = 0 and
+ * T_cap in {0, T}. */
+typedef struct {
+    int32_t L, B, H, T, d;
+    int32_t t0, T_cap;
+} cg_shape;
+
+/* Codec parameters.
+ *   backend  : CG_BLOCK_UNIFORM, CG_KIVI or CG_NONE
+ *   group    : gauge group g (Sec. 3, R = d/g groups per head); g in {8,16,32,64,128}, d % g == 0
+ *   bits     : 2, 3, 4, 6 or 8 (Sec. 4.3 bit settings; ignored by CG_NONE)
+ *   block    : a power of two >= 8 with d % block == 0 and block*bits % 8 == 0;
+ *              block-uniform: channels per block; KIVI: the key token-group length and
+ *              the value channel-group length
+ *   residual : KIVI full-precision window length R >= 0 (ignored otherwise)           */
+typedef struct {
+    int32_t backend;
+    int32_t group, bits, block, residual;
+} cg_params;
+
+/* Byte counts of the three output buffers for (shape, params): codes, scales and the KIVI
+ * residual (0 when the backend has none). Closed form of the layouts above (the measured
+ * bytes behind the paper's actual bits/value, Appendix metric table). Host-only; launches
+ * nothing. Returns CG_EINVAL on invalid arguments, CG_ERANGE on size_t overflow. */
+int cg_packed_bytes(const cg_shape* shape, const cg_params* params,
+                    size_t* codes_bytes, size_t* scales_bytes, size_t* residual_bytes);
+
+/* Encode (Sec. 3: Z = G X, B_c = C(Z)). Reads kv_bf16 [L][2][B][H][T][d] and gauges,
+ * writes the codes / scales / residual ranges that this shape covers (bytes outside them
+ * are left untouched). out_residual may be NULL unless the backend is CG_KIVI with
+ * T - n_q > 0; out_scales may be NULL for CG_NONE. All pointers must be 16-byte aligned.
+ * Non-finite inputs and fp16 overflow set device status bits (cg_get_status). */
+int cg_encode(const cg_shape* shape, const cg_params* params,
+              const void* kv_bf16, const float* gauges,
+              void* out_codes, void* out_scales, void* out_residual, void* stream);
+
+/* Decode (Sec. 3: Zhat = D(B_c), Xhat = G^{-1} Zhat with G^{-1} = G^T, Sec. 4.1). Reads
+ * the buffers written by cg_encode for the same params and writes out_kv_bf16
+ * [L][2][B][H][T][d] (the recovered cache restored before attention, Fig. 1). KIVI's
+ * residual tokens are copied back verbatim. Pointers 16-byte aligned. */
+int cg_decode(const cg_shape* shape, const cg_params* params,
+              const void* codes, const void* scales, const void* residual,
+              const float* gauges, void* out_kv_bf16, void* stream);
+
+/* Synchronizes `stream`, returns the accumulated CG_FLAG_* bits of the current device in
+ * *device_flags and clears them. Returns CG_ECUDA if the synchronize fails. */
+int cg_get_status(void* stream, int32_t* device_flags);
+
+/* Message for the most recent failing call on this host thread ("" if none). The pointer
+ * stays valid until the next library call on the same thread. */
+const char* cg_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CODECGAUGE_H */

@@ -1,0 +1,587 @@
+/*
+ * cg_oracle.c -- CPU oracle for the Codec-Gauge encode/decode path (arxiv 2607.20538).
+ *
+ * TEST INFRASTRUCTURE ONLY. Only the tests, the smoke check and the benchmark's CPU
+ * baseline leg load this library. The product path (libcodecgauge) never calls it, and
+ * the two share no source, header, table or helper.
+ *
+ * Plain, slow and direct: every function writes out the definition it cites, with no
+ * blocking, fusion or reordering. Arithmetic precision:
+ *   - gauge-space values z are fp32 (Sec. 4.3: the paper hands the backend FP32
+ *     transformed tensors); each z_i is the left-to-right chain acc = fmaf(G[i][j], x_j,
+ *     acc) over j = 0..g-1 starting from +0 -- a reading of Z = G X (Sec. 3 encode
+ *     equation) that fixes the summation order so that fp32 ranges are reproducible;
+ *   - the quantizer (Sec. 4.3 "asymmetric min/max") works in fp32 with fp16 scale/zero;
+ *   - decode (Sec. 3: Zhat = D(B_c), Xhat = G^{-1} Zhat, and G^{-1} = G^T by Sec. 4.1)
+ *     is evaluated in fp64 and returned as fp64.
+ * Compiled without fast-math and with -ffp-contract=off, so every operation below is
+ * the single IEEE operation it reads as.
+ *
+ * Status of the pins (tests/test_oracle_pins.py): every exported function is pinned
+ * against closed forms, brute force, worked examples or library routines; none is
+ * "parity unpinned".
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* ---- interface structs (same field layout as the library's; restated here) ---- */
+typedef struct { int32_t L, B, H, T, d, t0, T_cap; } cgo_shape;
+typedef struct { int32_t backend, group, bits, block, residual; } cgo_params;
+
+enum { CGO_BU = 0, CGO_KIVI = 1, CGO_NONE = 2 };
+enum { CGO_OK = 0, CGO_EINVAL = -1, CGO_EUNSUP = -2, CGO_ERANGE = -4 };
+enum { CGO_FLAG_NONFINITE = 1, CGO_FLAG_FP16_OVERFLOW = 2 };
+
+/* ------------------------------------------------------------------------------ */
+/* IEEE conversions, written from the format definitions                          */
+/* ------------------------------------------------------------------------------ */
+
+/* binary32 -> binary16, round to nearest, ties to even (IEEE 754 default rounding). */
+uint16_t cgo_f32_to_f16(float f)
+{
+    uint32_t x;
+    memcpy(&x, &f, 4);
+    uint32_t sign = (x >> 16) & 0x8000u;
+    uint32_t e32 = (x >> 23) & 0xffu;
+    uint32_t man = x & 0x7fffffu;
+    if (e32 == 0xffu) return (uint16_t)(sign | 0x7c00u | (man ? 0x200u : 0u));
+    if (e32 == 0u) return (uint16_t)sign; /* fp32 subnormals are far below half's range */
+    uint32_t sig = man | 0x800000u;       /* 24-bit significand, value = sig * 2^(e32-150) */
+    int32_t e16 = (int32_t)e32 - 127 + 15;
+    if (e16 >= 1) {
+        /* normal half: keep 11 significant bits, drop 13 */
+        uint32_t q = sig >> 13, rem = sig & 0x1fffu;
+        if (rem > 0x1000u || (rem == 0x1000u && (q & 1u))) q++;
+        if (q == 0x800u) { q = 0x400u; e16++; }
+        if (e16 >= 31) return (uint16_t)(sign | 0x7c00u);
+        return (uint16_t)(sign | ((uint32_t)e16 << 10) | (q & 0x3ffu));
+    }
+    /* subnormal half: unit 2^-24, q = sig * 2^(e32-150+24) = sig >> (126 - e32) */
+    uint32_t shift = 126u - e32; /* >= 14 here */
+    if (shift > 25u) return (uint16_t)sign;
+    uint32_t q = sig >> shift, rem = sig & ((1u << shift) - 1u), half = 1u << (shift - 1u);
+    if (rem > half || (rem == half && (q & 1u))) q++;
+    return (uint16_t)(sign | q); /* q == 0x400 lands on the smallest normal exactly */
+}
+
+float cgo_f16_to_f32(uint16_t h)
+{
+    uint32_t sign = (uint32_t)(h & 0x8000u) << 16;
+    uint32_t e = (h >> 10) & 0x1fu, m = h & 0x3ffu;
+    float v;
+    if (e == 0u) {
+        v = ldexpf((float)m, -24);
+    } else if (e == 31u) {
+        v = m ? NAN : INFINITY;
+    } else {
+        v = ldexpf((float)(m | 0x400u), (int)e - 25);
+    }
+    uint32_t bits;
+    memcpy(&bits, &v, 4);
+    bits |= sign;
+    memcpy(&v, &bits, 4);
+    return v;
+}
+
+float cgo_bf16_to_f32(uint16_t b)
+{
+    uint32_t bits = (uint32_t)b << 16;
+    float v;
+    memcpy(&v, &bits, 4);
+    return v;
+}
+
+/* ------------------------------------------------------------------------------ */
+/* Sizes and the KIVI split                                                        */
+/* ------------------------------------------------------------------------------ */
+
+static int valid_bits(int b) { return b == 2 || b == 3 || b == 4 || b == 6 || b == 8; }
+
+/* KIVI split (Sec. 4.3 KIVI-style path with a full-precision window): quantized tokens
+ * form whole token groups of length `block`; the newest T - n_q >= residual tokens stay
+ * raw. */
+int64_t cgo_kivi_nq(int64_t T, int64_t R, int64_t Gt)
+{
+    if (T <= R) return 0;
+    return ((T - R) / Gt) * Gt;
+}
+
+static int check_args(const cgo_shape* s, const cgo_params* p)
+{
+    if (!s || !p) return CGO_EINVAL;
+    if (s->L < 1 || s->B < 1 || s->H < 1 || s->T < 0 || s->d < 1) return CGO_EINVAL;
+    int g = p->group;
+    if (!(g == 8 || g == 16 || g == 32 || g == 64 || g == 128)) return CGO_EINVAL;
+    if (s->d % g) return CGO_EINVAL;
+    if (p->backend == CGO_BU) {
+        if (!valid_bits(p->bits) || p->block < 1 || s->d % p->block || (p->block * p->bits) % 8)
+            return CGO_EINVAL;
+    } else if (p->backend == CGO_KIVI) {
+        if (!valid_bits(p->bits) || p->block < 1 || s->d % p->block || (p->block * p->bits) % 8 ||
+            p->residual < 0)
+            return CGO_EINVAL;
+        if (s->t0 != 0 || (s->T_cap != 0 && s->T_cap != s->T)) return CGO_EUNSUP;
+    } else if (p->backend != CGO_NONE) {
+        return CGO_EINVAL;
+    }
+    if (s->t0 < 0 || s->T_cap < 0) return CGO_EINVAL;
+    if (s->T_cap != 0 && s->t0 + s->T > s->T_cap) return CGO_EINVAL;
+    return CGO_OK;
+}
+
+static int64_t tcap_of(const cgo_shape* s) { return s->T_cap ? s->T_cap : (int64_t)s->t0 + s->T; }
+
+/* Measured bytes of each buffer (Appendix metric table: actual bits/value = measured
+ * bytes / represented values), one count per stored item of the layouts. */
+int cgo_packed_bytes(const cgo_shape* s, const cgo_params* p, int64_t* codes, int64_t* scales,
+                     int64_t* resid)
+{
+    int rc = check_args(s, p);
+    if (rc) return rc;
+    int64_t units = (int64_t)s->L * 2 * s->B * s->H;
+    int64_t d = s->d;
+    if (p->backend == CGO_BU) {
+        int64_t tc = tcap_of(s), nb = d / p->block, pay = (int64_t)p->block * p->bits / 8;
+        *codes = units * tc * nb * pay;
+        *scales = units * tc * nb * 4;
+        *resid = 0;
+    } else if (p->backend == CGO_KIVI) {
+        int64_t nq = cgo_kivi_nq(s->T, p->residual, p->block);
+        int64_t per_lbh_key = (nq / p->block) * d * ((int64_t)p->block * p->bits / 8);
+        int64_t per_lbh_val = nq * (d / p->block) * ((int64_t)p->block * p->bits / 8);
+        int64_t lbh = (int64_t)s->L * s->B * s->H;
+        *codes = lbh * (per_lbh_key + per_lbh_val);
+        *scales = lbh * ((nq / p->block) * d + nq * (d / p->block)) * 4;
+        *resid = units * ((int64_t)s->T - nq) * d * 2;
+    } else {
+        *codes = units * tcap_of(s) * d * 4;
+        *scales = 0;
+        *resid = 0;
+    }
+    return CGO_OK;
+}
+
+/* ------------------------------------------------------------------------------ */
+/* Gauge application, quantizer, packing                                           */
+/* ------------------------------------------------------------------------------ */
+
+/* Z = G X for one token (Sec. 3): z[r*g + i] = sum_j G_r[i][j] x[r*g + j], as the fp32
+ * chain stated in the file header. Gh points at this (l, s, h)'s R gauges. */
+static void gauge_apply_f32(const float* Gh, const float* x, float* z, int d, int g)
+{
+    for (int r = 0; r < d / g; r++) {
+        const float* Gr = Gh + (size_t)r * g * g;
+        for (int i = 0; i < g; i++) {
+            float acc = 0.0f;
+            for (int j = 0; j < g; j++) acc = fmaf(Gr[(size_t)i * g + j], x[r * g + j], acc);
+            z[r * g + i] = acc;
+        }
+    }
+}
+
+/* Xhat = G^T Zhat for one token (Sec. 3 decode equation with G^{-1} = G^T, Sec. 4.1),
+ * in fp64: xh[r*g + i] = sum_j G_r[j][i] zh[r*g + j]. */
+static void gauge_inverse_f64(const float* Gh, const double* zh, double* xh, int d, int g)
+{
+    for (int r = 0; r < d / g; r++) {
+        const float* Gr = Gh + (size_t)r * g * g;
+        for (int i = 0; i < g; i++) {
+            double acc = 0.0;
+            for (int j = 0; j < g; j++) acc += (double)Gr[(size_t)j * g + i] * zh[r * g + j];
+            xh[r * g + i] = acc;
+        }
+    }
+}
+
+/* Asymmetric min/max quantizer over one block of n fp32 values (Sec. 4.3). Writes the
+ * fp16 scale and zero, the codes, and optionally the near-boundary flag of each value
+ * (pre-rounding value within 1e-4 steps of a half-integer). Returns status bits. */
+static int quantize_block(const float* v, int n, int stride, int bits, uint16_t* s16_out,
+                          uint16_t* m16_out, uint8_t* q_out, uint8_t* flag_out, int flag_stride)
+{
+    float mn = v[0], mx = v[0];
+    for (int k = 1; k < n; k++) {
+        float a = v[(size_t)k * stride];
+        if (a < mn) mn = a;
+        if (a > mx) mx = a;
+    }
+    const float qmax = (float)((1 << bits) - 1);
+    float s32 = (mx - mn) / qmax;
+    uint16_t s16 = cgo_f32_to_f16(s32), m16 = cgo_f32_to_f16(mn);
+    int st = 0;
+    if ((s16 & 0x7fffu) == 0x7c00u || (m16 & 0x7fffu) == 0x7c00u) st |= CGO_FLAG_FP16_OVERFLOW;
+    float s = cgo_f16_to_f32(s16), m = cgo_f16_to_f32(m16);
+    for (int k = 0; k < n; k++) {
+        uint8_t q = 0, fl = 0;
+        if (s != 0.0f) {
+            float t = (v[(size_t)k * stride] - m) / s;
+            float r = rintf(t); /* round half to even under the default rounding mode */
+            if (r < 0.0f) r = 0.0f;
+            if (r > qmax) r = qmax;
+            if (!(r == r)) r = 0.0f; /* inf scale: t is NaN or 0 */
+            q = (uint8_t)r;
+            float frac = t - floorf(t);
+            if (fabsf(frac - 0.5f) < 1e-4f) fl = 1;
+        }
+        q_out[k] = q;
+        if (flag_out) flag_out[(size_t)k * flag_stride] = fl;
+    }
+    *s16_out = s16;
+    *m16_out = m16;
+    return st;
+}
+
+/* Little-endian bit stream: code k occupies bits [k*bits, (k+1)*bits). */
+static void pack_codes(const uint8_t* q, int n, int bits, uint8_t* out)
+{
+    memset(out, 0, (size_t)n * bits / 8);
+    for (int k = 0; k < n; k++)
+        for (int b = 0; b < bits; b++)
+            if ((q[k] >> b) & 1) {
+                int pos = k * bits + b;
+                out[pos >> 3] |= (uint8_t)(1u << (pos & 7));
+            }
+}
+
+static void unpack_codes(const uint8_t* in, int n, int bits, uint8_t* q)
+{
+    for (int k = 0; k < n; k++) {
+        unsigned v = 0;
+        for (int b = 0; b < bits; b++) {
+            int pos = k * bits + b;
+            v |= (unsigned)((in[pos >> 3] >> (pos & 7)) & 1u) << b;
+        }
+        q[k] = (uint8_t)v;
+    }
+}
+
+void cgo_pack(const uint8_t* q, int n, int bits, uint8_t* out) { pack_codes(q, n, bits, out); }
+void cgo_unpack(const uint8_t* in, int n, int bits, uint8_t* q) { unpack_codes(in, n, bits, q); }
+
+static int has_nonfinite(const uint16_t* x, int64_t n)
+{
+    for (int64_t k = 0; k < n; k++)
+        if (((x[k] >> 7) & 0xffu) == 0xffu) return 1;
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------ */
+/* Work split over independent units (the gauge never mixes l, s, b, h: Sec. 3)     */
+/* ------------------------------------------------------------------------------ */
+
+typedef struct {
+    const cgo_shape* s;
+    const cgo_params* p;
+    const uint16_t* x;
+    const float* G;
+    uint8_t* codes;
+    uint16_t* scales;
+    uint16_t* resid;
+    float* z_out;
+    uint8_t* flag_out;
+    const uint8_t* in_codes;
+    const uint16_t* in_scales;
+    const uint16_t* in_resid;
+    double* xhat;
+    int64_t n_units;
+    int64_t next;
+    int status;
+    pthread_mutex_t mu;
+    void (*fn)(void* ctx, int64_t unit);
+} pool_t;
+
+static void* pool_worker(void* arg)
+{
+    pool_t* P = (pool_t*)arg;
+    for (;;) {
+        pthread_mutex_lock(&P->mu);
+        int64_t u = P->next++;
+        pthread_mutex_unlock(&P->mu);
+        if (u >= P->n_units) break;
+        P->fn(P, u);
+    }
+    return NULL;
+}
+
+static void run_pool(pool_t* P, int nthreads)
+{
+    if (nthreads < 1) nthreads = 1;
+    if (nthreads > 256) nthreads = 256;
+    pthread_mutex_init(&P->mu, NULL);
+    P->next = 0;
+    if (nthreads == 1) {
+        pool_worker(P);
+    } else {
+        pthread_t th[256];
+        for (int i = 0; i < nthreads; i++) pthread_create(&th[i], NULL, pool_worker, P);
+        for (int i = 0; i < nthreads; i++) pthread_join(th[i], NULL);
+    }
+    pthread_mutex_destroy(&P->mu);
+}
+
+static void add_status(pool_t* P, int st)
+{
+    if (!st) return;
+    pthread_mutex_lock(&P->mu);
+    P->status |= st;
+    pthread_mutex_unlock(&P->mu);
+}
+
+/* ---- block-uniform / none: one unit = (l, s, b, h) ---- */
+
+static void bu_encode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group;
+    int64_t h = u % s->H, sidx = (u / ((int64_t)s->H * s->B)) % 2, l = u / ((int64_t)s->H * s->B * 2);
+    const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+    int64_t tc = tcap_of(s);
+    float* x = (float*)malloc(sizeof(float) * d);
+    float* z = (float*)malloc(sizeof(float) * d);
+    uint8_t* q = (uint8_t*)malloc(d > 0 ? (size_t)d : 1);
+    int st = 0;
+    for (int64_t t = 0; t < s->T; t++) {
+        const uint16_t* xr = P->x + ((size_t)u * s->T + t) * d;
+        if (has_nonfinite(xr, d)) st |= CGO_FLAG_NONFINITE;
+        for (int c = 0; c < d; c++) x[c] = cgo_bf16_to_f32(xr[c]);
+        gauge_apply_f32(Gh, x, z, d, g);
+        int64_t th = s->t0 + t;
+        if (P->z_out) memcpy(P->z_out + ((size_t)u * s->T + t) * d, z, sizeof(float) * d);
+        if (p->backend == CGO_NONE) {
+            memcpy((float*)P->codes + ((size_t)u * tc + th) * d, z, sizeof(float) * d);
+            continue;
+        }
+        int nb = d / p->block, pay = p->block * p->bits / 8;
+        for (int b = 0; b < nb; b++) {
+            uint16_t s16, m16;
+            uint8_t* fl = P->flag_out ? P->flag_out + ((size_t)u * s->T + t) * d + (size_t)b * p->block : NULL;
+            st |= quantize_block(z + b * p->block, p->block, 1, p->bits, &s16, &m16, q, fl, 1);
+            size_t blk_index = ((size_t)u * tc + th) * nb + b;
+            pack_codes(q, p->block, p->bits, P->codes + blk_index * pay);
+            P->scales[blk_index * 2 + 0] = s16;
+            P->scales[blk_index * 2 + 1] = m16;
+        }
+    }
+    add_status(P, st);
+    free(x);
+    free(z);
+    free(q);
+}
+
+static void bu_decode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group;
+    int64_t h = u % s->H, sidx = (u / ((int64_t)s->H * s->B)) % 2, l = u / ((int64_t)s->H * s->B * 2);
+    const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+    int64_t tc = tcap_of(s);
+    double* zh = (double*)malloc(sizeof(double) * d);
+    uint8_t* q = (uint8_t*)malloc((size_t)d);
+    for (int64_t t = 0; t < s->T; t++) {
+        int64_t th = s->t0 + t;
+        if (p->backend == CGO_NONE) {
+            const float* zr = (const float*)P->in_codes + ((size_t)u * tc + th) * d;
+            for (int c = 0; c < d; c++) zh[c] = (double)zr[c];
+        } else {
+            int nb = d / p->block, pay = p->block * p->bits / 8;
+            for (int b = 0; b < nb; b++) {
+                size_t blk_index = ((size_t)u * tc + th) * nb + b;
+                unpack_codes(P->in_codes + blk_index * pay, p->block, p->bits, q);
+                double sc = (double)cgo_f16_to_f32(P->in_scales[blk_index * 2 + 0]);
+                double mz = (double)cgo_f16_to_f32(P->in_scales[blk_index * 2 + 1]);
+                for (int k = 0; k < p->block; k++) zh[b * p->block + k] = (double)q[k] * sc + mz;
+            }
+        }
+        gauge_inverse_f64(Gh, zh, P->xhat + ((size_t)u * s->T + t) * d, d, g);
+    }
+    free(zh);
+    free(q);
+}
+
+/* ---- KIVI: one unit = (l, b, h); keys and values handled together ---- */
+
+static void kivi_offsets(const cgo_shape* s, const cgo_params* p, int64_t l, int64_t bh, int64_t* key_codes,
+                         int64_t* val_codes, int64_t* key_scales, int64_t* val_scales)
+{
+    int64_t d = s->d, Gt = p->block, nq = cgo_kivi_nq(s->T, p->residual, Gt);
+    int64_t pay = Gt * p->bits / 8;
+    int64_t key_per = (nq / Gt) * d * pay, val_per = nq * (d / Gt) * pay;
+    int64_t BH = (int64_t)s->B * s->H;
+    int64_t layer_codes = BH * (key_per + val_per);
+    *key_codes = l * layer_codes + bh * key_per;
+    *val_codes = l * layer_codes + BH * key_per + bh * val_per;
+    int64_t ks_per = (nq / Gt) * d, vs_per = nq * (d / Gt);
+    int64_t layer_scales = BH * (ks_per + vs_per);
+    *key_scales = l * layer_scales + bh * ks_per;
+    *val_scales = l * layer_scales + BH * ks_per + bh * vs_per;
+}
+
+static void kivi_encode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group, Gt = p->block, bits = p->bits, pay = Gt * bits / 8;
+    int64_t T = s->T, nq = cgo_kivi_nq(T, p->residual, Gt);
+    int64_t bh = u % ((int64_t)s->B * s->H), l = u / ((int64_t)s->B * s->H), h = bh % s->H, b = bh / s->H;
+    int64_t kc, vc, ks, vs;
+    kivi_offsets(s, p, l, bh, &kc, &vc, &ks, &vs);
+    float* x = (float*)malloc(sizeof(float) * d);
+    float* Z = (float*)malloc(sizeof(float) * (size_t)(nq > 0 ? nq : 1) * d);
+    uint8_t* q = (uint8_t*)malloc((size_t)(Gt > d ? Gt : d));
+    int st = 0;
+    for (int sidx = 0; sidx < 2; sidx++) {
+        int64_t unit5 = ((l * 2 + sidx) * s->B + b) * s->H + h; /* index of (l,s,b,h) */
+        const uint16_t* X = P->x + (size_t)unit5 * T * d;
+        const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+        if (has_nonfinite(X, T * d)) st |= CGO_FLAG_NONFINITE;
+        /* gauge-space tensor of the quantized tokens */
+        for (int64_t t = 0; t < nq; t++) {
+            for (int c = 0; c < d; c++) x[c] = cgo_bf16_to_f32(X[t * d + c]);
+            gauge_apply_f32(Gh, x, Z + (size_t)t * d, d, g);
+        }
+        if (P->z_out) memcpy(P->z_out + (size_t)unit5 * T * d, Z, sizeof(float) * (size_t)nq * d);
+        if (sidx == 0) {
+            /* keys: one range per channel over each group of Gt tokens (KIVI per-channel keys) */
+            for (int64_t tg = 0; tg < nq / Gt; tg++)
+                for (int c = 0; c < d; c++) {
+                    uint16_t s16, m16;
+                    uint8_t* fl = P->flag_out ? P->flag_out + ((size_t)unit5 * T + tg * Gt) * d + c : NULL;
+                    st |= quantize_block(Z + (size_t)tg * Gt * d + c, Gt, d, bits, &s16, &m16, q, fl, d);
+                    int64_t idx = tg * d + c;
+                    pack_codes(q, Gt, bits, P->codes + kc + idx * pay);
+                    P->scales[(ks + idx) * 2 + 0] = s16;
+                    P->scales[(ks + idx) * 2 + 1] = m16;
+                }
+        } else {
+            /* values: one range per token over each group of Gt channels (KIVI per-token values) */
+            int nb = d / Gt;
+            for (int64_t t = 0; t < nq; t++)
+                for (int blk = 0; blk < nb; blk++) {
+                    uint16_t s16, m16;
+                    uint8_t* fl = P->flag_out ? P->flag_out + ((size_t)unit5 * T + t) * d + (size_t)blk * Gt : NULL;
+                    st |= quantize_block(Z + (size_t)t * d + (size_t)blk * Gt, Gt, 1, bits, &s16, &m16, q, fl, 1);
+                    int64_t idx = t * nb + blk;
+                    pack_codes(q, Gt, bits, P->codes + vc + idx * pay);
+                    P->scales[(vs + idx) * 2 + 0] = s16;
+                    P->scales[(vs + idx) * 2 + 1] = m16;
+                }
+        }
+        /* residual window: the newest T - nq tokens, raw bf16 */
+        if (T - nq > 0)
+            memcpy(P->resid + (size_t)unit5 * (T - nq) * d, X + (size_t)nq * d, sizeof(uint16_t) * (size_t)(T - nq) * d);
+    }
+    add_status(P, st);
+    free(x);
+    free(Z);
+    free(q);
+}
+
+static void kivi_decode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group, Gt = p->block, bits = p->bits, pay = Gt * bits / 8;
+    int64_t T = s->T, nq = cgo_kivi_nq(T, p->residual, Gt);
+    int64_t bh = u % ((int64_t)s->B * s->H), l = u / ((int64_t)s->B * s->H), h = bh % s->H, b = bh / s->H;
+    int64_t kc, vc, ks, vs;
+    kivi_offsets(s, p, l, bh, &kc, &vc, &ks, &vs);
+    double* Zh = (double*)malloc(sizeof(double) * (size_t)(nq > 0 ? nq : 1) * d);
+    uint8_t* q = (uint8_t*)malloc((size_t)(Gt > d ? Gt : d));
+    for (int sidx = 0; sidx < 2; sidx++) {
+        int64_t unit5 = ((l * 2 + sidx) * s->B + b) * s->H + h;
+        const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+        if (sidx == 0) {
+            for (int64_t tg = 0; tg < nq / Gt; tg++)
+                for (int c = 0; c < d; c++) {
+                    int64_t idx = tg * d + c;
+                    unpack_codes(P->in_codes + kc + idx * pay, Gt, bits, q);
+                    double sc = (double)cgo_f16_to_f32(P->in_scales[(ks + idx) * 2 + 0]);
+                    double mz = (double)cgo_f16_to_f32(P->in_scales[(ks + idx) * 2 + 1]);
+                    for (int k = 0; k < Gt; k++) Zh[(size_t)(tg * Gt + k) * d + c] = (double)q[k] * sc + mz;
+                }
+        } else {
+            int nb = d / Gt;
+            for (int64_t t = 0; t < nq; t++)
+                for (int blk = 0; blk < nb; blk++) {
+                    int64_t idx = t * nb + blk;
+                    unpack_codes(P->in_codes + vc + idx * pay, Gt, bits, q);
+                    double sc = (double)cgo_f16_to_f32(P->in_scales[(vs + idx) * 2 + 0]);
+                    double mz = (double)cgo_f16_to_f32(P->in_scales[(vs + idx) * 2 + 1]);
+                    for (int k = 0; k < Gt; k++) Zh[(size_t)t * d + (size_t)blk * Gt + k] = (double)q[k] * sc + mz;
+                }
+        }
+        double* out = P->xhat + (size_t)unit5 * T * d;
+        for (int64_t t = 0; t < nq; t++) gauge_inverse_f64(Gh, Zh + (size_t)t * d, out + (size_t)t * d, d, g);
+        for (int64_t t = nq; t < T; t++)
+            for (int c = 0; c < d; c++)
+                out[(size_t)t * d + c] = (double)cgo_bf16_to_f32(P->in_resid[((size_t)unit5 * (T - nq) + (t - nq)) * d + c]);
+    }
+    free(Zh);
+    free(q);
+}
+
+/* ------------------------------------------------------------------------------ */
+/* Exported entry points                                                           */
+/* ------------------------------------------------------------------------------ */
+
+/* Encode (Sec. 3: Z = G X, B_c = C(Z)). z_out (fp32 [L][2][B][H][T][d]) and flag_out (u8,
+ * same layout: 1 = pre-rounding value within 1e-4 steps of a rounding boundary) are
+ * optional. Returns a CGO_* code; *status_out receives the CGO_FLAG_* bits. */
+int cgo_encode(const cgo_shape* s, const cgo_params* p, const uint16_t* x, const float* G, uint8_t* codes,
+               uint16_t* scales, uint16_t* resid, float* z_out, uint8_t* flag_out, int nthreads,
+               int32_t* status_out)
+{
+    int rc = check_args(s, p);
+    if (rc) return rc;
+    pool_t P;
+    memset(&P, 0, sizeof P);
+    P.s = s; P.p = p; P.x = x; P.G = G; P.codes = codes; P.scales = scales; P.resid = resid;
+    P.z_out = z_out; P.flag_out = flag_out;
+    if (p->backend == CGO_KIVI) {
+        P.n_units = (int64_t)s->L * s->B * s->H;
+        P.fn = kivi_encode_unit;
+    } else {
+        P.n_units = (int64_t)s->L * 2 * s->B * s->H;
+        P.fn = bu_encode_unit;
+    }
+    run_pool(&P, nthreads);
+    if (status_out) *status_out = P.status;
+    return CGO_OK;
+}
+
+/* Decode (Sec. 3: Zhat = D(B_c), Xhat = G^T Zhat). xhat: fp64 [L][2][B][H][T][d]. */
+int cgo_decode(const cgo_shape* s, const cgo_params* p, const uint8_t* codes, const uint16_t* scales,
+               const uint16_t* resid, const float* G, double* xhat, int nthreads)
+{
+    int rc = check_args(s, p);
+    if (rc) return rc;
+    pool_t P;
+    memset(&P, 0, sizeof P);
+    P.s = s; P.p = p; P.G = G; P.in_codes = codes; P.in_scales = scales; P.in_resid = resid; P.xhat = xhat;
+    if (p->backend == CGO_KIVI) {
+        P.n_units = (int64_t)s->L * s->B * s->H;
+        P.fn = kivi_decode_unit;
+    } else {
+        P.n_units = (int64_t)s->L * 2 * s->B * s->H;
+        P.fn = bu_decode_unit;
+    }
+    run_pool(&P, nthreads);
+    return CGO_OK;
+}
+
+/* The gauge-space value of one coordinate, exposed so that tests can pin the chain. */
+float cgo_gauge_coord(const float* Grow, const float* x, int g)
+{
+    float acc = 0.0f;
+    for (int j = 0; j < g; j++) acc = fmaf(Grow[j], x[j], acc);
+    return acc;
+}
