@@ -1,0 +1,336 @@
+"""Benchmark: encode + decode of a KV cache through libcodecgauge on GB300.
+
+One step = one pass of the hot path over the workload: cg_encode (gauge rotation, block
+ranges, scales, codes, packing) then cg_decode (unpacking, dequantization, inverse gauge)
+of the whole cache, with inputs resident in HBM (1 GiB of bf16 for the Llama-3-8B-shaped
+cache, larger than the 129 MB L2, so no flush is needed between steps).
+
+value  = (bf16 bytes encoded + bf16 bytes decoded) / (encode + decode time), GB/s
+e2e    = the same through the C ABI with host buffers: pinned host -> device copy of the
+         cache, encode, decode, device -> pinned host copy of the recovered cache.
+roofline: the slower of the two kernels; algorithmic bytes per launch / its average
+         CUDA-event duration, against the measured copy bandwidth.
+
+Multi-GPU (torchrun): every rank encodes/decodes its own cache of the same shape (the
+units (l, s, b, h) are independent; no collective on the data path), weak scaling.
+--impl reference times the CPU oracle on the host cores on a bounded sample.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "encode/decode KV GB/s (bf16 bytes) and % of HBM roofline at 1 GB300"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev_index: int):
+        self.dev = dev_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.dev}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        time.sleep(0.05)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [v.strip() for v in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _kernel_traffic(kind: str):
+    """ncu DRAM bytes per launch recorded in profiles/traffic.json, or None when the kernel
+    source changed since the counters were taken."""
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        rec = json.load(open(p))[kind]
+    except Exception:
+        return None
+    src = os.path.join(ROOT, "paper_2607_20538_gb300", "csrc", rec["source"])
+    try:
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except Exception:
+        return None
+    return rec["bytes_per_launch"] if h == rec["source_sha"] else None
+
+
+def cpu_sample(w, G, seconds=12.0, nthreads=None):
+    """Time the oracle (as it stands) on whole (l, s, b, h) units of the workload."""
+    import numpy as np
+
+    import oracle
+    from paper_2607_20538_gb300 import synth
+    nthreads = nthreads or os.cpu_count() or 1
+    done_bytes, t_total, layers = 0, 0.0, 0
+    for l in range(w.L):
+        sub = w.replace(L=1)
+        x = np.stack([np.stack([np.stack([np.stack([synth.kv_unit(w, l, s, b, h) for h in range(w.H)])
+                                          for b in range(w.B)]) for s in range(2)])])
+        Gl = np.ascontiguousarray(G[l:l + 1])
+        t0 = time.perf_counter()
+        r = oracle.encode(sub.shape, sub.params, x, Gl, nthreads=nthreads)
+        oracle.decode(sub.shape, sub.params, r["codes"], r["scales"], r["residual"], Gl, nthreads=nthreads)
+        t_total += time.perf_counter() - t0
+        done_bytes += 2 * x.nbytes
+        layers += 1
+        if t_total >= seconds:
+            break
+    return {"value": done_bytes / t_total / 1e9, "unit": "GB/s", "cores": nthreads, "kind": "oracle",
+            "sample": f"encode+decode of {layers} of {w.L} layers of the {w.name} cache "
+                      f"({layers * 2 * w.B * w.H} (l,s,b,h) units, {done_bytes // 2} bf16 bytes), "
+                      f"{t_total:.1f} s on {nthreads} threads"}
+
+
+def run_reference(args):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    from paper_2607_20538_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    G = synth.gauges(w)
+    cores = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        cpu_sample(w.replace(L=1), G, seconds=0.0, nthreads=cores)
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        vals.append(cpu_sample(w, G, seconds=1.0, nthreads=cores))
+    el = time.perf_counter() - t0
+    v = statistics.median(x["value"] for x in vals)
+    line = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(el / args.steps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": {"workload": w.name},
+            "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                             "sample": vals[-1]["sample"]},
+            "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_cuda(args):
+    import numpy as np
+    import torch
+
+    import paper_2607_20538_gb300 as cg
+    from paper_2607_20538_gb300 import synth
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+    w = synth.WORKLOADS[args.workload]
+    shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
+    nc, ns, nr = cg.packed_bytes(shape, params)
+    x = synth.kv_cache(w, threads=max(4, (os.cpu_count() or 8) // max(ws, 1)))
+    G = synth.gauges(w)
+    dx = torch.from_numpy(x.reshape(-1).view(np.int16)).to(dev)
+    dG = torch.from_numpy(G.reshape(-1)).to(dev)
+    codes, scales, resid = cg.alloc_outputs(shape, params, device=dev)
+    out = torch.empty_like(dx)
+    stream = torch.cuda.current_stream()
+    n_bf16 = x.nbytes
+    g_bytes = G.nbytes
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    flags = cg.get_status()
+    if flags:
+        raise RuntimeError(f"device status flags {flags} after warm-up")
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = Clocks(dev if ws == 1 else local)
+    clocks.start()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    enc_ms = [e[0].elapsed_time(e[1]) for e in evs]
+    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
+    if ws > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_step = total_ms / args.steps
+    value = ws * 2 * n_bf16 / (ms_step * 1e-3) / 1e9
+    enc_avg, dec_avg = statistics.mean(enc_ms), statistics.mean(dec_ms)
+    enc_alg = n_bf16 + nc + ns + nr + g_bytes
+    dec_alg = nc + ns + nr + g_bytes + n_bf16
+    peak, peak_kind = _peaks()
+    if dec_avg >= enc_avg:
+        dom, dom_ms, dom_alg = "decode", dec_avg, dec_alg
+    else:
+        dom, dom_ms, dom_alg = "encode", enc_avg, enc_alg
+    achieved = dom_alg / (dom_ms * 1e-3) / 1e9
+
+    # end to end through the C ABI with host buffers
+    hx = torch.from_numpy(x.reshape(-1).view(np.int16)).pin_memory()
+    hout = torch.empty_like(hx).pin_memory()
+    e2e_steps = max(3, min(args.steps, 20))
+
+    def e2e_step():
+        dx.copy_(hx, non_blocking=True)
+        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
+        hout.copy_(out, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    e2e_val = ws * 2 * n_bf16 / (e2e_ms * 1e-3) / 1e9
+    if ws > 1:
+        t = torch.tensor([e2e_val], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MIN)
+        e2e_val = float(t.item()) * 1.0
+    flags = cg.get_status()
+    if flags:
+        raise RuntimeError(f"device status flags {flags} after the timed region")
+
+    if rank == 0:
+        launches_per_step = 2 if w.backend != 1 else 2 * (1 + 1 + 1)
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms_step, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
+                       "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
+                       "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
+                       "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
+                       "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"},
+            "encode_gbs": round(n_bf16 / (enc_avg * 1e-3) / 1e9, 2),
+            "decode_gbs": round(n_bf16 / (dec_avg * 1e-3) / 1e9, 2),
+            "encode_ms": round(enc_avg, 5), "decode_ms": round(dec_avg, 5),
+            "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 2), "peak": peak,
+                         "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
+                         "traffic": _kernel_traffic(dom), "alg_bytes_per_launch": dom_alg,
+                         "enc_frac": round(enc_alg / (enc_avg * 1e-3) / 1e9 / peak, 4),
+                         "dec_frac": round(dec_alg / (dec_avg * 1e-3) / 1e9 / peak, 4)},
+            "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": n_bf16,
+                    "d2h_bytes_per_step": n_bf16},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk,
+        }
+        if not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_sample(w, G, seconds=args.cpu_seconds)
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
+    ap.add_argument("--workload", default="llama3_8b")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_cuda(args)
+
+
+if __name__ == "__main__":
+    main()

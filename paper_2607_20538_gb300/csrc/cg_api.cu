@@ -1,0 +1,379 @@
+// cg_api.cu -- the extern "C" boundary of libcodecgauge: argument validation, the
+// closed-form byte counts, kernel selection, the device status word and error strings.
+// Declarations and the full contract: include/codecgauge.h.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include "cg_launch.h"
+#include "cg_tc.h"
+
+namespace cg {
+
+__device__ int32_t g_status_word = 0;
+
+namespace {
+
+thread_local std::string t_err;
+
+int fail(int code, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_err = buf;
+    return code;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(CG_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+bool pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
+bool valid_bits(int b) { return b == 2 || b == 3 || b == 4 || b == 6 || b == 8; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Address of this device's status word (looked up once per device).
+int status_ptr(int32_t** out) {
+    static std::mutex mu;
+    static int32_t* ptrs[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return fail(CG_EUNSUPPORTED, "device ordinal %d out of range", dev);
+    std::lock_guard<std::mutex> lk(mu);
+    if (!ptrs[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_status_word);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+        ptrs[dev] = static_cast<int32_t*>(p);
+    }
+    *out = ptrs[dev];
+    return CG_OK;
+}
+
+struct Sizes {
+    int64_t tcap, nq, nb, pay;
+    size_t codes, scales, resid;
+    int64_t layer_codes, layer_scales, key_codes_per_bh, key_scales_per_bh, val_codes_per_bh, val_scales_per_bh;
+};
+
+bool mul_ok(size_t a, size_t b, size_t* out) {
+    if (a && b > SIZE_MAX / a) return false;
+    *out = a * b;
+    return true;
+}
+
+int validate(const cg_shape* sh, const cg_params* p, Sizes* z) {
+    if (!sh || !p) return fail(CG_EINVAL, "null shape or params");
+    if (sh->L < 1 || sh->B < 1 || sh->H < 1 || sh->T < 0 || sh->d < 1)
+        return fail(CG_EINVAL, "shape needs L,B,H,d >= 1 and T >= 0 (got L=%d B=%d H=%d T=%d d=%d)", sh->L, sh->B,
+                    sh->H, sh->T, sh->d);
+    if (!(sh->d == 32 || sh->d == 64 || sh->d == 128 || sh->d == 256))
+        return fail(CG_EUNSUPPORTED, "head dim d=%d: supported d is 32, 64, 128 or 256", sh->d);
+    const int g = p->group;
+    if (!(g == 8 || g == 16 || g == 32 || g == 64 || g == 128) || sh->d % g)
+        return fail(CG_EINVAL, "group=%d: must be one of 8,16,32,64,128 and divide d=%d", g, sh->d);
+    if (sh->t0 < 0 || sh->T_cap < 0) return fail(CG_EINVAL, "t0 and T_cap must be >= 0");
+    if (p->backend == CG_BLOCK_UNIFORM || p->backend == CG_KIVI) {
+        if (!valid_bits(p->bits)) return fail(CG_EINVAL, "bits=%d: must be 2, 3, 4, 6 or 8", p->bits);
+        if (!pow2(p->block) || p->block < 8 || sh->d % p->block)
+            return fail(CG_EINVAL, "block=%d: must be a power of two >= 8 that divides d=%d", p->block, sh->d);
+        if ((p->block * p->bits) % 8) return fail(CG_EINVAL, "block*bits must be a whole number of bytes");
+    } else if (p->backend != CG_NONE) {
+        return fail(CG_EINVAL, "unknown backend %d", p->backend);
+    }
+    if (p->backend == CG_KIVI) {
+        if (p->residual < 0) return fail(CG_EINVAL, "residual must be >= 0");
+        if (sh->t0 != 0 || (sh->T_cap != 0 && sh->T_cap != sh->T))
+            return fail(CG_EUNSUPPORTED, "KIVI append into a history (t0 > 0 or T_cap != T) is not provided");
+        if (key_simt_smem(sh->d, g, p->block, p->bits) > 200 * 1024)
+            return fail(CG_EUNSUPPORTED, "KIVI key group of %d tokens x d=%d does not fit one CTA", p->block, sh->d);
+    }
+    const int64_t tcap = sh->T_cap ? sh->T_cap : (int64_t)sh->t0 + sh->T;
+    if ((int64_t)sh->t0 + sh->T > tcap) return fail(CG_EINVAL, "t0 + T = %lld exceeds T_cap = %lld",
+                                                     (long long)sh->t0 + sh->T, (long long)tcap);
+    if ((int64_t)sh->L * 2 * sh->H > 65535 || (int64_t)sh->L * sh->B * sh->H > 65535)
+        return fail(CG_ERANGE, "L*2*H and L*B*H must be <= 65535");
+    const int64_t units = (int64_t)sh->L * 2 * sh->B * sh->H;
+    z->tcap = tcap;
+    z->nq = 0;
+    z->resid = 0;
+    z->layer_codes = z->layer_scales = z->key_codes_per_bh = z->key_scales_per_bh = 0;
+    z->val_codes_per_bh = z->val_scales_per_bh = 0;
+    size_t rows, tmp;
+    if (!mul_ok((size_t)units, (size_t)tcap, &rows)) return fail(CG_ERANGE, "size overflow");
+    if (p->backend == CG_NONE) {
+        z->nb = 0;
+        z->pay = 0;
+        if (!mul_ok(rows, (size_t)sh->d * 4, &z->codes)) return fail(CG_ERANGE, "size overflow");
+        z->scales = 0;
+    } else if (p->backend == CG_BLOCK_UNIFORM) {
+        z->nb = sh->d / p->block;
+        z->pay = (int64_t)p->block * p->bits / 8;
+        if (!mul_ok(rows, (size_t)(z->nb * z->pay), &z->codes)) return fail(CG_ERANGE, "size overflow");
+        if (!mul_ok(rows, (size_t)z->nb * 4, &z->scales)) return fail(CG_ERANGE, "size overflow");
+    } else {
+        const int64_t Gt = p->block, d = sh->d;
+        z->nq = kivi_nq(sh->T, p->residual, Gt);
+        z->nb = d / Gt;
+        z->pay = Gt * p->bits / 8;
+        z->key_codes_per_bh = (z->nq / Gt) * d * z->pay;
+        z->val_codes_per_bh = z->nq * z->nb * z->pay;
+        z->key_scales_per_bh = (z->nq / Gt) * d;
+        z->val_scales_per_bh = z->nq * z->nb;
+        const int64_t BH = (int64_t)sh->B * sh->H;
+        z->layer_codes = BH * (z->key_codes_per_bh + z->val_codes_per_bh);
+        z->layer_scales = BH * (z->key_scales_per_bh + z->val_scales_per_bh);
+        if (!mul_ok((size_t)sh->L, (size_t)z->layer_codes, &z->codes)) return fail(CG_ERANGE, "size overflow");
+        if (!mul_ok((size_t)sh->L, (size_t)z->layer_scales * 4, &z->scales)) return fail(CG_ERANGE, "size overflow");
+        if (!mul_ok((size_t)units, (size_t)(sh->T - z->nq) * d * 2, &z->resid)) return fail(CG_ERANGE, "size overflow");
+    }
+    if (!mul_ok(rows, (size_t)sh->d * 2, &tmp)) return fail(CG_ERANGE, "size overflow");
+    return CG_OK;
+}
+
+// Row map for the block-uniform / none history layout [L][2][B][H][T_cap][...].
+void bu_maps(const cg_shape* sh, const Sizes& z, int64_t rowbytes, int64_t rowscales, RowMap* cm, RowMap* sm) {
+    const int64_t tc = z.tcap;
+    cm->sT = rowbytes;
+    cm->sH = tc * rowbytes;
+    cm->sB = (int64_t)sh->H * cm->sH;
+    cm->sS = (int64_t)sh->B * cm->sB;
+    cm->sL = 2 * cm->sS;
+    cm->base = (int64_t)sh->t0 * rowbytes;
+    sm->sT = rowscales;
+    sm->sH = tc * rowscales;
+    sm->sB = (int64_t)sh->H * sm->sH;
+    sm->sS = (int64_t)sh->B * sm->sB;
+    sm->sL = 2 * sm->sS;
+    sm->base = (int64_t)sh->t0 * rowscales;
+}
+
+// Row map for KIVI values: codes [B][H][n_q][d/blk][pay] after the layer's key part.
+void kivi_value_maps(const cg_shape* sh, const Sizes& z, RowMap* cm, RowMap* sm) {
+    const int64_t BH = (int64_t)sh->B * sh->H;
+    cm->sT = z.nb * z.pay;
+    cm->sH = z.val_codes_per_bh;
+    cm->sB = (int64_t)sh->H * cm->sH;
+    cm->sS = 0;
+    cm->sL = z.layer_codes;
+    cm->base = BH * z.key_codes_per_bh;
+    sm->sT = z.nb;
+    sm->sH = z.val_scales_per_bh;
+    sm->sB = (int64_t)sh->H * sm->sH;
+    sm->sS = 0;
+    sm->sL = z.layer_scales;
+    sm->base = BH * z.key_scales_per_bh;
+}
+
+RowArgs row_args(const cg_shape* sh, const cg_params* p, int32_t* status) {
+    RowArgs a{};
+    a.status = status;
+    a.L = sh->L;
+    a.B = sh->B;
+    a.H = sh->H;
+    a.d = sh->d;
+    a.g = p->group;
+    a.bits = p->bits;
+    a.blk = p->block;
+    a.s_lo = 0;
+    a.s_n = 2;
+    a.T_x = sh->T;
+    a.t_count = sh->T;
+    a.none_mode = p->backend == CG_NONE;
+    return a;
+}
+
+KeyArgs key_args(const cg_shape* sh, const cg_params* p, const Sizes& z, int32_t* status) {
+    KeyArgs k{};
+    k.status = status;
+    k.L = sh->L;
+    k.B = sh->B;
+    k.H = sh->H;
+    k.d = sh->d;
+    k.g = p->group;
+    k.bits = p->bits;
+    k.Gt = p->block;
+    k.T = sh->T;
+    k.nq = z.nq;
+    k.layer_codes = z.layer_codes;
+    k.layer_scales = z.layer_scales;
+    k.key_codes_per_bh = z.key_codes_per_bh;
+    k.key_scales_per_bh = z.key_scales_per_bh;
+    return k;
+}
+
+}  // namespace
+}  // namespace cg
+
+using namespace cg;
+
+extern "C" {
+
+const char* cg_last_error(void) { return t_err.c_str(); }
+
+int cg_packed_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes, size_t* scales_bytes,
+                    size_t* residual_bytes) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate(shape, params, &z);
+    if (rc) return rc;
+    if (codes_bytes) *codes_bytes = z.codes;
+    if (scales_bytes) *scales_bytes = z.scales;
+    if (residual_bytes) *residual_bytes = z.resid;
+    return CG_OK;
+}
+
+int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf16, const float* gauges,
+              void* out_codes, void* out_scales, void* out_residual, void* stream) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate(shape, params, &z);
+    if (rc) return rc;
+    const bool kivi = params->backend == CG_KIVI, none = params->backend == CG_NONE;
+    if (shape->T == 0) return CG_OK;
+    if (!kv_bf16 || !gauges) return fail(CG_EINVAL, "null kv or gauges pointer");
+    if (z.codes && !out_codes) return fail(CG_EINVAL, "null out_codes");
+    if (!none && z.scales && !out_scales) return fail(CG_EINVAL, "null out_scales");
+    if (kivi && z.resid && !out_residual) return fail(CG_EINVAL, "null out_residual");
+    if (!aligned16(kv_bf16) || !aligned16(gauges) || !aligned16(out_codes) || !aligned16(out_scales) ||
+        !aligned16(out_residual))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    RowArgs a = row_args(shape, params, status);
+    a.x = static_cast<const uint16_t*>(kv_bf16);
+    a.G = gauges;
+    a.codes = static_cast<uint8_t*>(out_codes);
+    a.scales = static_cast<uint32_t*>(out_scales);
+    if (!kivi) {
+        bu_maps(shape, z, none ? (int64_t)shape->d * 4 : z.nb * z.pay, z.nb, &a.cmap, &a.smap);
+        if (!none && tc_row_encode_eligible(a)) {
+            e = tc_launch_row_encode(a, st);
+        } else {
+            e = launch_row_encode_simt(a, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "row encode launch");
+        return CG_OK;
+    }
+    if (z.nq > 0) {
+        KeyArgs k = key_args(shape, params, z, status);
+        k.x = a.x;
+        k.G = gauges;
+        k.codes = a.codes;
+        k.scales = a.scales;
+        e = launch_key_encode_simt(k, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI key encode launch");
+        a.s_lo = 1;
+        a.s_n = 1;
+        a.t_count = z.nq;
+        kivi_value_maps(shape, z, &a.cmap, &a.smap);
+        e = launch_row_encode_simt(a, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI value encode launch");
+    }
+    if (shape->T - z.nq > 0) {
+        ResidArgs r{};
+        r.src = a.x;
+        r.dst = static_cast<uint16_t*>(out_residual);
+        r.units = (int64_t)shape->L * 2 * shape->B * shape->H;
+        r.T = shape->T;
+        r.nq = z.nq;
+        r.d = shape->d;
+        r.to_residual = 1;
+        e = launch_residual_copy(r, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI residual copy launch");
+    }
+    return CG_OK;
+}
+
+int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes, const void* scales,
+              const void* residual, const float* gauges, void* out_kv_bf16, void* stream) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate(shape, params, &z);
+    if (rc) return rc;
+    const bool kivi = params->backend == CG_KIVI, none = params->backend == CG_NONE;
+    if (shape->T == 0) return CG_OK;
+    if (!out_kv_bf16 || !gauges) return fail(CG_EINVAL, "null output or gauges pointer");
+    if (z.codes && !codes) return fail(CG_EINVAL, "null codes");
+    if (!none && z.scales && !scales) return fail(CG_EINVAL, "null scales");
+    if (kivi && z.resid && !residual) return fail(CG_EINVAL, "null residual");
+    if (!aligned16(codes) || !aligned16(scales) || !aligned16(residual) || !aligned16(gauges) ||
+        !aligned16(out_kv_bf16))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaSuccess;
+    RowArgs a = row_args(shape, params, status);
+    a.out = static_cast<uint16_t*>(out_kv_bf16);
+    a.G = gauges;
+    a.codes = const_cast<uint8_t*>(static_cast<const uint8_t*>(codes));
+    a.scales = const_cast<uint32_t*>(static_cast<const uint32_t*>(scales));
+    if (!kivi) {
+        bu_maps(shape, z, none ? (int64_t)shape->d * 4 : z.nb * z.pay, z.nb, &a.cmap, &a.smap);
+        if (!none && tc_row_decode_eligible(a)) {
+            e = tc_launch_row_decode(a, st);
+        } else {
+            e = launch_row_decode_simt(a, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "row decode launch");
+        return CG_OK;
+    }
+    if (z.nq > 0) {
+        KeyArgs k = key_args(shape, params, z, status);
+        k.out = a.out;
+        k.G = gauges;
+        k.codes = a.codes;
+        k.scales = a.scales;
+        e = launch_key_decode_simt(k, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI key decode launch");
+        a.s_lo = 1;
+        a.s_n = 1;
+        a.t_count = z.nq;
+        kivi_value_maps(shape, z, &a.cmap, &a.smap);
+        e = launch_row_decode_simt(a, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI value decode launch");
+    }
+    if (shape->T - z.nq > 0) {
+        ResidArgs r{};
+        r.src = static_cast<const uint16_t*>(residual);
+        r.dst = a.out;
+        r.units = (int64_t)shape->L * 2 * shape->B * shape->H;
+        r.T = shape->T;
+        r.nq = z.nq;
+        r.d = shape->d;
+        r.to_residual = 0;
+        e = launch_residual_copy(r, st);
+        if (e != cudaSuccess) return cuda_fail(e, "KIVI residual copy launch");
+    }
+    return CG_OK;
+}
+
+int cg_get_status(void* stream, int32_t* device_flags) {
+    t_err.clear();
+    if (!device_flags) return fail(CG_EINVAL, "null device_flags");
+    int32_t* status = nullptr;
+    int rc = status_ptr(&status);
+    if (rc) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    int32_t v = 0;
+    e = cudaMemcpy(&v, status, sizeof v, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "read status");
+    const int32_t zero = 0;
+    e = cudaMemcpy(status, &zero, sizeof zero, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "clear status");
+    *device_flags = v;
+    return CG_OK;
+}
+
+}  // extern "C"

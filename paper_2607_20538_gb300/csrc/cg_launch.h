@@ -1,0 +1,62 @@
+// cg_launch.h -- internal launcher interface between the C ABI (cg_api.cu) and the kernel
+// translation units. Not installed; not part of the public ABI.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "cg_common.cuh"
+
+namespace cg {
+
+// One "row" = one token vector of one (l, s, b, h) unit. Row kernels process, for each
+// (l, s, h) that shares a gauge, the rows (b, t) for b < B and t < t_count.
+struct RowArgs {
+    const uint16_t* x;      // encode: bf16 input [L][2][B][H][T_x][d]
+    uint16_t* out;          // decode: bf16 output [L][2][B][H][T_x][d]
+    const float* G;         // [L][2][H][d/g][g][g]
+    uint8_t* codes;         // packed codes (or fp32 z for CG_NONE)
+    uint32_t* scales;       // half2 {s, m} per block
+    int32_t* status;
+    int L, B, H, d, g, bits, blk;
+    int s_lo, s_n;          // cache types handled: s in [s_lo, s_lo + s_n)
+    int64_t T_x;            // tokens per unit in the dense x / out tensor
+    int64_t t_count;        // tokens processed per unit
+    int none_mode;          // 1 = CG_NONE (codes hold fp32 z rows)
+    RowMap cmap;            // byte offset of a row's codes
+    RowMap smap;            // u32 index of a row's first block scale
+};
+
+// KIVI keys: one CTA per (l, b, h, token group); per-channel ranges over Gt tokens.
+struct KeyArgs {
+    const uint16_t* x;      // encode input  [L][2][B][H][T][d] (keys are s = 0)
+    uint16_t* out;          // decode output [L][2][B][H][T][d]
+    const float* G;
+    uint8_t* codes;         // whole codes buffer
+    uint32_t* scales;       // whole scales buffer
+    int32_t* status;
+    int L, B, H, d, g, bits, Gt;
+    int64_t T, nq;
+    int64_t layer_codes, layer_scales;  // bytes / u32 per layer
+    int64_t key_codes_per_bh, key_scales_per_bh;
+};
+
+struct ResidArgs {
+    const uint16_t* src;
+    uint16_t* dst;
+    int64_t units;          // L*2*B*H
+    int64_t T, nq, d;
+    int to_residual;        // 1: x -> residual window, 0: residual window -> out
+};
+
+cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st);
+cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st);
+cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st);
+cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st);
+cudaError_t launch_residual_copy(const ResidArgs& a, cudaStream_t st);
+
+// Shared-memory bytes the SIMT kernels need (0 = shape not supported by them).
+size_t row_simt_smem(int d, int g);
+size_t key_simt_smem(int d, int g, int Gt, int bits);
+
+}  // namespace cg

@@ -1,0 +1,450 @@
+// cg_simt.cu -- CUDA-core kernels of the encode/decode path.
+//
+// These kernels evaluate the gauge rotation Z = G X (Sec. 3) exactly as the library's
+// quantization rule defines it: each z_i is the fp32 fused multiply-add chain over the
+// group's channels in increasing order, so scales, zeros and codes are reproducible to
+// the bit. They serve every shape the library accepts and are the launch choice where a
+// tile of tokens is too small or the group too small for the tensor-core kernels.
+//
+// Thread mapping (row kernels): one warp per token row; lane owns channels c = lane + 32k.
+// The (l, s, h) gauge set sits in shared memory; one CTA handles 64 rows (b, t) that
+// share it.
+#include "cg_launch.h"
+
+namespace cg {
+namespace {
+
+constexpr int kRowThreads = 256;
+constexpr int kRowWarps = kRowThreads / 32;
+constexpr int kRowsPerCta = 64;
+
+__device__ __forceinline__ float seg_min(float v, int seg) {
+    for (int off = seg >> 1; off >= 1; off >>= 1) v = fminf(v, __shfl_xor_sync(0xffffffffu, v, off));
+    return v;
+}
+__device__ __forceinline__ float seg_max(float v, int seg) {
+    for (int off = seg >> 1; off >= 1; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
+    return v;
+}
+
+// Extract the b-bit code that starts at bit p of a little-endian word stream.
+__device__ __forceinline__ uint32_t extract_code(const uint32_t* w, int p, int bits) {
+    int wi = p >> 5, off = p & 31;
+    uint32_t v = w[wi] >> off;
+    if (off + bits > 32) v |= w[wi + 1] << (32 - off);
+    return v & ((1u << bits) - 1u);
+}
+
+// Word w of the little-endian stream in which code c sits at bits [c*bits, (c+1)*bits).
+__device__ __forceinline__ uint32_t pack_word(const uint8_t* q, int w, int bits) {
+    int bit0 = w * 32, c0 = bit0 / bits, c1 = (bit0 + 31) / bits;
+    uint32_t word = 0;
+    for (int c = c0; c <= c1; c++) {
+        int p = c * bits - bit0;
+        uint32_t v = q[c];
+        word |= p >= 0 ? (v << p) : (v >> (-p));
+    }
+    return word;
+}
+
+// ------------------------------------------------------------------------------------
+// Row encode: Z = G X, then per-token block min/max quantization and packing (or the raw
+// fp32 Z for the no-compression rows).
+// ------------------------------------------------------------------------------------
+template <int NR>
+__global__ void __launch_bounds__(kRowThreads) row_encode_kernel(RowArgs a) {
+    constexpr int d = NR * 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int g = a.g;
+    float* Gs = reinterpret_cast<float*>(smem);  // Gs[r][jj][i] = G_r[i][jj]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* xs = reinterpret_cast<float*>(smem + (size_t)d * g * 4) + warp * d;
+    uint8_t* qs = smem + (size_t)d * g * 4 + (size_t)kRowWarps * d * 4 + warp * d;
+    uint32_t* sm = reinterpret_cast<uint32_t*>(smem + (size_t)d * g * 4 + (size_t)kRowWarps * d * 5) + warp * 32;
+
+    const int y = blockIdx.y;
+    const int h = y % a.H;
+    const int s = a.s_lo + (y / a.H) % a.s_n;
+    const int l = y / (a.H * a.s_n);
+    const float* Gsrc = a.G + ((int64_t)(l * 2 + s) * a.H + h) * (int64_t)d * g;
+    for (int e = threadIdx.x; e < d * g; e += kRowThreads) {
+        int r = e / (g * g), rem = e - r * g * g, i = rem / g, jj = rem - i * g;
+        Gs[r * g * g + jj * g + i] = __ldg(Gsrc + e);
+    }
+    __syncthreads();
+
+    const int64_t rows = (int64_t)a.B * a.t_count;
+    const int64_t r0 = (int64_t)blockIdx.x * kRowsPerCta;
+    const int bits = a.bits, blk = a.blk;
+    const int qmax = (1 << bits) - 1;
+    const float qmaxf = (float)qmax;
+    int32_t flag = 0;
+
+    for (int rr = warp; rr < kRowsPerCta; rr += kRowWarps) {
+        const int64_t row = r0 + rr;
+        if (row >= rows) break;
+        const int b = (int)(row / a.t_count);
+        const int64_t t = row - (int64_t)b * a.t_count;
+        const uint16_t* xr = a.x + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d;
+        float z[NR];
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            uint32_t xb = xr[lane + 32 * k];
+            if (bf16_nonfinite(xb)) flag |= CG_FLAG_NONFINITE_INPUT;
+            xs[lane + 32 * k] = bf16_bits_to_float(xb);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k, r = c / g, i = c - r * g;
+            const float* Gcol = Gs + r * g * g + i;
+            const float* xg = xs + r * g;
+            float acc = 0.0f;
+            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], xg[jj], acc);
+            z[k] = acc;
+        }
+        const int64_t coff = a.cmap.at(l, s, b, h, t);
+        if (a.none_mode) {
+            float* zr = reinterpret_cast<float*>(a.codes + coff);
+#pragma unroll
+            for (int k = 0; k < NR; k++) zr[lane + 32 * k] = z[k];
+            __syncwarp();
+            continue;
+        }
+        // block ranges: segments of min(blk, 32) lanes per register, then registers
+        const int seg = blk < 32 ? blk : 32;
+        const int per = blk > 32 ? blk / 32 : 1;
+        float mn[NR], mx[NR];
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            mn[k] = seg_min(z[k], seg);
+            mx[k] = seg_max(z[k], seg);
+        }
+        if (per > 1) {
+#pragma unroll
+            for (int k = 0; k < NR; k++) {
+                const int k0 = (k / per) * per;
+                float a0 = mn[k0], a1 = mx[k0];
+                for (int kk = 1; kk < per; kk++) {
+                    a0 = fminf(a0, mn[k0 + kk]);
+                    a1 = fmaxf(a1, mx[k0 + kk]);
+                }
+                mn[k] = a0;
+                mx[k] = a1;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k;
+            const uint32_t sz = scale_zero(mn[k], mx[k], qmaxf, &flag);
+            const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
+            qs[c] = (uint8_t)quant_code(z[k], sc, mz, qmax);
+            if ((c % blk) == 0) sm[c / blk] = sz;
+        }
+        __syncwarp();
+        uint32_t* cw = reinterpret_cast<uint32_t*>(a.codes + coff);
+        const int nw = d * bits / 32;
+        for (int w = lane; w < nw; w += 32) cw[w] = pack_word(qs, w, bits);
+        const int nb = d / blk;
+        if (lane < nb) a.scales[a.smap.at(l, s, b, h, t) + lane] = sm[lane];
+        __syncwarp();
+    }
+    if (flag) raise_flag(a.status, flag);
+}
+
+// ------------------------------------------------------------------------------------
+// Row decode: unpack, dequantize zhat = q*s + m, then Xhat = G^T Zhat, bf16 store.
+// ------------------------------------------------------------------------------------
+template <int NR>
+__global__ void __launch_bounds__(kRowThreads) row_decode_kernel(RowArgs a) {
+    constexpr int d = NR * 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int g = a.g;
+    float* Gs = reinterpret_cast<float*>(smem);  // Gs[r][jj][i] = G_r[jj][i]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* zs = reinterpret_cast<float*>(smem + (size_t)d * g * 4) + warp * d;
+    uint32_t* cwS = reinterpret_cast<uint32_t*>(smem + (size_t)d * g * 4 + (size_t)kRowWarps * d * 4) + warp * (d / 4 + 4);
+    uint32_t* sm = reinterpret_cast<uint32_t*>(smem + (size_t)d * g * 4 + (size_t)kRowWarps * d * 4 +
+                                               (size_t)kRowWarps * (d / 4 + 4) * 4) + warp * 32;
+
+    const int y = blockIdx.y;
+    const int h = y % a.H;
+    const int s = a.s_lo + (y / a.H) % a.s_n;
+    const int l = y / (a.H * a.s_n);
+    const float* Gsrc = a.G + ((int64_t)(l * 2 + s) * a.H + h) * (int64_t)d * g;
+    for (int e = threadIdx.x; e < d * g; e += kRowThreads) Gs[e] = __ldg(Gsrc + e);
+    __syncthreads();
+
+    const int64_t rows = (int64_t)a.B * a.t_count;
+    const int64_t r0 = (int64_t)blockIdx.x * kRowsPerCta;
+    const int bits = a.bits, blk = a.blk;
+
+    for (int rr = warp; rr < kRowsPerCta; rr += kRowWarps) {
+        const int64_t row = r0 + rr;
+        if (row >= rows) break;
+        const int b = (int)(row / a.t_count);
+        const int64_t t = row - (int64_t)b * a.t_count;
+        const int64_t coff = a.cmap.at(l, s, b, h, t);
+        if (a.none_mode) {
+            const float* zr = reinterpret_cast<const float*>(a.codes + coff);
+#pragma unroll
+            for (int k = 0; k < NR; k++) zs[lane + 32 * k] = zr[lane + 32 * k];
+        } else {
+            const uint32_t* cw = reinterpret_cast<const uint32_t*>(a.codes + coff);
+            const int nw = d * bits / 32, nb = d / blk;
+            for (int w = lane; w < nw; w += 32) cwS[w] = cw[w];
+            if (lane < nb) sm[lane] = a.scales[a.smap.at(l, s, b, h, t) + lane];
+            __syncwarp();
+#pragma unroll
+            for (int k = 0; k < NR; k++) {
+                const int c = lane + 32 * k;
+                const uint32_t q = extract_code(cwS, c * bits, bits);
+                const uint32_t sz = sm[c / blk];
+                zs[c] = fmaf((float)q, h2f_bits(sz & 0xffffu), h2f_bits(sz >> 16));
+            }
+        }
+        __syncwarp();
+        uint16_t* orow = a.out + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d;
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k, r = c / g, i = c - r * g;
+            const float* Gcol = Gs + r * g * g + i;
+            const float* zg = zs + r * g;
+            float acc = 0.0f;
+            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], zg[jj], acc);
+            orow[c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+        }
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------------------------------
+// KIVI keys: per-channel ranges over a group of Gt tokens (one CTA per (l, b, h, group)).
+// ------------------------------------------------------------------------------------
+template <int NR>
+__global__ void __launch_bounds__(kRowThreads) key_encode_kernel(KeyArgs a) {
+    constexpr int d = NR * 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int g = a.g, Gt = a.Gt, bits = a.bits;
+    const int pay = Gt * bits / 8;
+    float* Gs = reinterpret_cast<float*>(smem);                          // transposed
+    float* Zs = reinterpret_cast<float*>(smem + (size_t)d * g * 4);      // [Gt][d]
+    float* xsAll = Zs + (size_t)Gt * d;                                  // [warps][d]
+    uint8_t* stage = reinterpret_cast<uint8_t*>(xsAll + kRowWarps * d);  // [d][pay]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float* xs = xsAll + warp * d;
+
+    const int64_t tg = blockIdx.x;
+    const int bh = blockIdx.y % (a.B * a.H), l = blockIdx.y / (a.B * a.H);
+    const int b = bh / a.H, h = bh % a.H;
+    const float* Gsrc = a.G + ((int64_t)(l * 2 + 0) * a.H + h) * (int64_t)d * g;
+    for (int e = threadIdx.x; e < d * g; e += kRowThreads) {
+        int r = e / (g * g), rem = e - r * g * g, i = rem / g, jj = rem - i * g;
+        Gs[r * g * g + jj * g + i] = __ldg(Gsrc + e);
+    }
+    __syncthreads();
+    int32_t flag = 0;
+    const uint16_t* X = a.x + ((((int64_t)(l * 2 + 0) * a.B + b) * a.H + h) * a.T + tg * Gt) * d;
+    for (int t = warp; t < Gt; t += kRowWarps) {
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            uint32_t xb = X[(int64_t)t * d + lane + 32 * k];
+            if (bf16_nonfinite(xb)) flag |= CG_FLAG_NONFINITE_INPUT;
+            xs[lane + 32 * k] = bf16_bits_to_float(xb);
+        }
+        __syncwarp();
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k, r = c / g, i = c - r * g;
+            const float* Gcol = Gs + r * g * g + i;
+            const float* xg = xs + r * g;
+            float acc = 0.0f;
+            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], xg[jj], acc);
+            Zs[(size_t)t * d + c] = acc;
+        }
+        __syncwarp();
+    }
+    __syncthreads();
+    const int qmax = (1 << bits) - 1;
+    const float qmaxf = (float)qmax;
+    const int64_t bhl = (int64_t)b * a.H + h;
+    for (int c = threadIdx.x; c < d; c += kRowThreads) {
+        float mn = Zs[c], mx = Zs[c];
+        for (int t = 1; t < Gt; t++) {
+            const float v = Zs[(size_t)t * d + c];
+            mn = fminf(mn, v);
+            mx = fmaxf(mx, v);
+        }
+        const uint32_t sz = scale_zero(mn, mx, qmaxf, &flag);
+        const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
+        uint8_t* st = stage + (size_t)c * pay;
+        uint64_t acc = 0;
+        int nacc = 0, nbytes = 0;
+        for (int t = 0; t < Gt; t++) {
+            acc |= (uint64_t)quant_code(Zs[(size_t)t * d + c], sc, mz, qmax) << nacc;
+            nacc += bits;
+            while (nacc >= 8) {
+                st[nbytes++] = (uint8_t)(acc & 0xffu);
+                acc >>= 8;
+                nacc -= 8;
+            }
+        }
+        a.scales[(int64_t)l * a.layer_scales + bhl * a.key_scales_per_bh + tg * d + c] = sz;
+    }
+    __syncthreads();
+    uint32_t* dst = reinterpret_cast<uint32_t*>(a.codes + (int64_t)l * a.layer_codes + bhl * a.key_codes_per_bh +
+                                                tg * (int64_t)d * pay);
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(stage);
+    for (int w = threadIdx.x; w < d * pay / 4; w += kRowThreads) dst[w] = src[w];
+    if (flag) raise_flag(a.status, flag);
+}
+
+template <int NR>
+__global__ void __launch_bounds__(kRowThreads) key_decode_kernel(KeyArgs a) {
+    constexpr int d = NR * 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int g = a.g, Gt = a.Gt, bits = a.bits;
+    const int pay = Gt * bits / 8;
+    float* Gs = reinterpret_cast<float*>(smem);                      // untransposed
+    float* Zs = reinterpret_cast<float*>(smem + (size_t)d * g * 4);  // [Gt][d]
+    uint8_t* stage = reinterpret_cast<uint8_t*>(Zs + (size_t)Gt * d);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    const int64_t tg = blockIdx.x;
+    const int bh = blockIdx.y % (a.B * a.H), l = blockIdx.y / (a.B * a.H);
+    const int b = bh / a.H, h = bh % a.H;
+    const int64_t bhl = (int64_t)b * a.H + h;
+    const float* Gsrc = a.G + ((int64_t)(l * 2 + 0) * a.H + h) * (int64_t)d * g;
+    for (int e = threadIdx.x; e < d * g; e += kRowThreads) Gs[e] = __ldg(Gsrc + e);
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(a.codes + (int64_t)l * a.layer_codes +
+                                                            bhl * a.key_codes_per_bh + tg * (int64_t)d * pay);
+    uint32_t* stw = reinterpret_cast<uint32_t*>(stage);
+    for (int w = threadIdx.x; w < d * pay / 4; w += kRowThreads) stw[w] = src[w];
+    __syncthreads();
+    for (int c = threadIdx.x; c < d; c += kRowThreads) {
+        const uint32_t sz = a.scales[(int64_t)l * a.layer_scales + bhl * a.key_scales_per_bh + tg * d + c];
+        const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
+        const uint8_t* st = stage + (size_t)c * pay;
+        for (int t = 0; t < Gt; t++) {
+            const int p = t * bits;
+            uint32_t v = st[p >> 3] >> (p & 7);
+            if ((p & 7) + bits > 8) v |= (uint32_t)st[(p >> 3) + 1] << (8 - (p & 7));
+            v &= (1u << bits) - 1u;
+            Zs[(size_t)t * d + c] = fmaf((float)v, sc, mz);
+        }
+    }
+    __syncthreads();
+    uint16_t* O = a.out + ((((int64_t)(l * 2 + 0) * a.B + b) * a.H + h) * a.T + tg * Gt) * d;
+    for (int t = warp; t < Gt; t += kRowWarps) {
+        const float* zr = Zs + (size_t)t * d;
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k, r = c / g, i = c - r * g;
+            const float* Gcol = Gs + r * g * g + i;
+            const float* zg = zr + r * g;
+            float acc = 0.0f;
+            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], zg[jj], acc);
+            O[(int64_t)t * d + c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
+        }
+    }
+}
+
+__global__ void residual_copy_kernel(ResidArgs a) {
+    const int64_t n16 = (a.T - a.nq) * a.d * 2 / 16;  // 16-byte chunks per unit
+    for (int64_t u = blockIdx.y; u < a.units; u += gridDim.y) {
+        const uint4* src;
+        uint4* dst;
+        if (a.to_residual) {
+            src = reinterpret_cast<const uint4*>(a.src + (u * a.T + a.nq) * a.d);
+            dst = reinterpret_cast<uint4*>(a.dst + u * (a.T - a.nq) * a.d);
+        } else {
+            src = reinterpret_cast<const uint4*>(a.src + u * (a.T - a.nq) * a.d);
+            dst = reinterpret_cast<uint4*>(a.dst + (u * a.T + a.nq) * a.d);
+        }
+        for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n16; i += (int64_t)gridDim.x * blockDim.x)
+            dst[i] = src[i];
+    }
+}
+
+}  // namespace
+
+size_t row_simt_smem(int d, int g) {
+    if (!(d == 32 || d == 64 || d == 128 || d == 256)) return 0;
+    size_t enc = (size_t)d * g * 4 + (size_t)kRowWarps * d * 5 + (size_t)kRowWarps * 32 * 4;
+    size_t dec = (size_t)d * g * 4 + (size_t)kRowWarps * d * 4 + (size_t)kRowWarps * (d / 4 + 4) * 4 +
+                 (size_t)kRowWarps * 32 * 4;
+    return enc > dec ? enc : dec;
+}
+
+size_t key_simt_smem(int d, int g, int Gt, int bits) {
+    if (!(d == 32 || d == 64 || d == 128 || d == 256)) return 0;
+    size_t pay = (size_t)Gt * bits / 8;
+    size_t enc = (size_t)d * g * 4 + (size_t)Gt * d * 4 + (size_t)kRowWarps * d * 4 + (size_t)d * pay;
+    return enc;
+}
+
+template <int NR>
+static cudaError_t row_encode_nr(const RowArgs& a, cudaStream_t st) {
+    size_t smem = row_simt_smem(a.d, a.g);
+    cudaError_t e = cudaFuncSetAttribute(row_encode_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((a.B * a.t_count + kRowsPerCta - 1) / kRowsPerCta), (unsigned)(a.L * a.s_n * a.H));
+    row_encode_kernel<NR><<<grid, kRowThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+template <int NR>
+static cudaError_t row_decode_nr(const RowArgs& a, cudaStream_t st) {
+    size_t smem = row_simt_smem(a.d, a.g);
+    cudaError_t e = cudaFuncSetAttribute(row_decode_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((a.B * a.t_count + kRowsPerCta - 1) / kRowsPerCta), (unsigned)(a.L * a.s_n * a.H));
+    row_decode_kernel<NR><<<grid, kRowThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+template <int NR>
+static cudaError_t key_encode_nr(const KeyArgs& a, cudaStream_t st) {
+    size_t smem = key_simt_smem(a.d, a.g, a.Gt, a.bits);
+    cudaError_t e = cudaFuncSetAttribute(key_encode_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)(a.nq / a.Gt), (unsigned)(a.L * a.B * a.H));
+    key_encode_kernel<NR><<<grid, kRowThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+template <int NR>
+static cudaError_t key_decode_nr(const KeyArgs& a, cudaStream_t st) {
+    size_t smem = key_simt_smem(a.d, a.g, a.Gt, a.bits);
+    cudaError_t e = cudaFuncSetAttribute(key_decode_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)(a.nq / a.Gt), (unsigned)(a.L * a.B * a.H));
+    key_decode_kernel<NR><<<grid, kRowThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+#define CG_NR_SWITCH(FN, d, ...)                      \
+    switch ((d) / 32) {                               \
+        case 1: return FN<1>(__VA_ARGS__);            \
+        case 2: return FN<2>(__VA_ARGS__);            \
+        case 4: return FN<4>(__VA_ARGS__);            \
+        case 8: return FN<8>(__VA_ARGS__);            \
+        default: return cudaErrorInvalidValue;        \
+    }
+
+cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_encode_nr, a.d, a, st) }
+cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_decode_nr, a.d, a, st) }
+cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_encode_nr, a.d, a, st) }
+cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_decode_nr, a.d, a, st) }
+
+cudaError_t launch_residual_copy(const ResidArgs& a, cudaStream_t st) {
+    const int64_t n16 = (a.T - a.nq) * a.d * 2 / 16;
+    if (n16 <= 0 || a.units <= 0) return cudaSuccess;
+    unsigned gx = (unsigned)((n16 + 255) / 256);
+    if (gx > 1024) gx = 1024;
+    dim3 grid(gx, (unsigned)(a.units < 65535 ? a.units : 65535));
+    residual_copy_kernel<<<grid, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace cg

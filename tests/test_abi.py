@@ -1,0 +1,88 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol the header
+declares, computes byte counts equal to the oracle's closed form, and rejects invalid
+arguments with the documented status before touching the device."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from paper_2607_20538_gb300 import synth
+
+cg = pytest.importorskip("paper_2607_20538_gb300")
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(cg.lib_path()):
+        from paper_2607_20538_gb300 import build
+        build.build()
+    return cg.load()
+
+
+def _declared_symbols():
+    names = set()
+    for f in os.listdir(os.path.join(ROOT, "include")):
+        if f.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", f)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"^\s*(?:const\s+)?\w+[\s\*]+(cg_\w+)\s*\(", src, flags=re.M))
+    return names
+
+
+def test_exports_every_declared_symbol(lib):
+    names = _declared_symbols()
+    assert {"cg_packed_bytes", "cg_encode", "cg_decode", "cg_get_status", "cg_last_error"} <= names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+@pytest.mark.parametrize("name", list(synth.WORKLOADS))
+def test_packed_bytes_match_oracle(lib, name):
+    w = synth.WORKLOADS[name]
+    assert cg.packed_bytes(cg.Shape(**w.shape), cg.Params(**w.params)) == oracle.packed_bytes(w.shape, w.params)
+    for backend in (0, 1, 2):
+        for T in (0, 1, 127, 128, 129, 300):
+            ww = w.replace(backend=backend, T=T, T_cap=0, L=2, B=2, H=3)
+            assert cg.packed_bytes(cg.Shape(**ww.shape), cg.Params(**ww.params)) == \
+                oracle.packed_bytes(ww.shape, ww.params)
+
+
+@pytest.mark.parametrize("bad", [
+    dict(group=12), dict(group=256), dict(bits=5), dict(bits=1), dict(block=24), dict(block=4),
+    dict(block=256), dict(backend=7), dict(d=48), dict(d=512), dict(T=-1), dict(L=0),
+    dict(block=8, bits=3, d=64, group=8, _ok=True),
+])
+def test_validation(lib, bad):
+    kw = dict(L=1, B=1, H=1, T=16, d=128, group=64, backend=0, bits=4, block=64, residual=0)
+    ok = bad.pop("_ok", False)
+    kw.update(bad)
+    shape = cg.Shape(L=kw["L"], B=kw["B"], H=kw["H"], T=kw["T"], d=kw["d"])
+    params = cg.Params(kw["backend"], kw["group"], kw["bits"], kw["block"], kw["residual"])
+    if ok:
+        cg.packed_bytes(shape, params)
+        return
+    with pytest.raises(cg.CodecGaugeError) as e:
+        cg.packed_bytes(shape, params)
+    assert e.value.code in (-1, -2)
+    assert lib.cg_last_error().decode()
+
+
+def test_pointer_checks_fail_before_device(lib):
+    shape = cg.Shape(L=1, B=1, H=1, T=4, d=64)
+    params = cg.Params(0, 16, 4, 32)
+    S, P = ctypes.byref(shape.c()), ctypes.byref(params.c())
+    assert lib.cg_encode(S, P, None, None, None, None, None, None) == -1
+    assert lib.cg_decode(S, P, None, None, None, None, None, None) == -1
+    assert lib.cg_encode(S, P, ctypes.c_void_p(0x1001), ctypes.c_void_p(0x2000), ctypes.c_void_p(0x3000),
+                         ctypes.c_void_p(0x4000), None, None) == -1
+    assert "aligned" in lib.cg_last_error().decode()
+    kp = cg.Params(1, 16, 4, 32, 8)
+    assert lib.cg_encode(ctypes.byref(cg.Shape(L=1, B=1, H=1, T=4, d=64, t0=2, T_cap=8).c()),
+                         ctypes.byref(kp.c()), None, None, None, None, None, None) == -2
+    assert lib.cg_get_status(None, None) == -1
+    # history overflow: t0 + T > T_cap
+    assert lib.cg_packed_bytes(ctypes.byref(cg.Shape(L=1, B=1, H=1, T=4, d=64, t0=6, T_cap=8).c()), P,
+                               None, None, None) == -1
