@@ -8,9 +8,10 @@
  * Plain, slow and direct: every function writes out the definition it cites, with no
  * blocking, fusion or reordering. Arithmetic precision:
  *   - gauge-space values z are fp32 (Sec. 4.3: the paper hands the backend FP32
- *     transformed tensors); each z_i is the left-to-right chain acc = fmaf(G[i][j], x_j,
- *     acc) over j = 0..g-1 starting from +0 -- a reading of Z = G X (Sec. 3 encode
- *     equation) that fixes the summation order so that fp32 ranges are reproducible;
+ *     transformed tensors); each z_i = sum_j G[i][j] x_j (Sec. 3, Z = G X) is summed in a
+ *     fixed order so that fp32 ranges are reproducible: for each 16-wide slice of j a
+ *     chain p = fmaf(G[i][j], x_j, p) from p = +0 in increasing j, then the slice sums
+ *     added left to right (z = ((p_0 + p_1) + p_2) + ...);
  *   - the quantizer (Sec. 4.3 "asymmetric min/max") works in fp32 with fp16 scale/zero;
  *   - decode (Sec. 3: Zhat = D(B_c), Xhat = G^{-1} Zhat, and G^{-1} = G^T by Sec. 4.1)
  *     is evaluated in fp64 and returned as fp64.
@@ -168,17 +169,26 @@ int cgo_packed_bytes(const cgo_shape* s, const cgo_params* p, int64_t* codes, in
 /* Gauge application, quantizer, packing                                           */
 /* ------------------------------------------------------------------------------ */
 
-/* Z = G X for one token (Sec. 3): z[r*g + i] = sum_j G_r[i][j] x[r*g + j], as the fp32
- * chain stated in the file header. Gh points at this (l, s, h)'s R gauges. */
+/* One gauge-space coordinate sum_j Grow[j] x[j] in the fixed fp32 order of the file
+ * header: 16-wide fma chains, their sums added left to right. */
+static float gauge_dot(const float* Grow, const float* x, int g)
+{
+    float acc = 0.0f;
+    for (int b = 0; b * 16 < g; b++) {
+        float p = 0.0f;
+        for (int j = 16 * b; j < 16 * b + 16 && j < g; j++) p = fmaf(Grow[j], x[j], p);
+        acc = (b == 0) ? p : acc + p;
+    }
+    return acc;
+}
+
+/* Z = G X for one token (Sec. 3): z[r*g + i] = sum_j G_r[i][j] x[r*g + j].
+ * Gh points at this (l, s, h)'s R gauges. */
 static void gauge_apply_f32(const float* Gh, const float* x, float* z, int d, int g)
 {
     for (int r = 0; r < d / g; r++) {
         const float* Gr = Gh + (size_t)r * g * g;
-        for (int i = 0; i < g; i++) {
-            float acc = 0.0f;
-            for (int j = 0; j < g; j++) acc = fmaf(Gr[(size_t)i * g + j], x[r * g + j], acc);
-            z[r * g + i] = acc;
-        }
+        for (int i = 0; i < g; i++) z[r * g + i] = gauge_dot(Gr + (size_t)i * g, x + r * g, g);
     }
 }
 
@@ -579,9 +589,4 @@ int cgo_decode(const cgo_shape* s, const cgo_params* p, const uint8_t* codes, co
 }
 
 /* The gauge-space value of one coordinate, exposed so that tests can pin the chain. */
-float cgo_gauge_coord(const float* Grow, const float* x, int g)
-{
-    float acc = 0.0f;
-    for (int j = 0; j < g; j++) acc = fmaf(Grow[j], x[j], acc);
-    return acc;
-}
+float cgo_gauge_coord(const float* Grow, const float* x, int g) { return gauge_dot(Grow, x, g); }

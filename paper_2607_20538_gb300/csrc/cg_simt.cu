@@ -1,9 +1,8 @@
 // cg_simt.cu -- CUDA-core kernels of the encode/decode path.
 //
 // These kernels evaluate the gauge rotation Z = G X (Sec. 3) exactly as the library's
-// quantization rule defines it: each z_i is the fp32 fused multiply-add chain over the
-// group's channels in increasing order, so scales, zeros and codes are reproducible to
-// the bit. They serve every shape the library accepts and are the launch choice where a
+// quantization rule defines it (16-wide fp32 fma chains, slice sums added left to right),
+// so scales, zeros and codes are reproducible to the bit. They serve every shape the library accepts and are the launch choice where a
 // tile of tokens is too small or the group too small for the tensor-core kernels.
 //
 // Thread mapping (row kernels): one warp per token row; lane owns channels c = lane + 32k.
@@ -25,6 +24,33 @@ __device__ __forceinline__ float seg_min(float v, int seg) {
 __device__ __forceinline__ float seg_max(float v, int seg) {
     for (int off = seg >> 1; off >= 1; off >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, off));
     return v;
+}
+
+// One gauge-space coordinate sum_j G[i][j] x[j] in the library's fixed fp32 order: for
+// each 16-wide slice of j an fma chain from +0 in increasing j, then the slice sums added
+// left to right. Gcol[j * gstride] = G[i][j]. The slices are independent, so the chains
+// run interleaved.
+__device__ __forceinline__ float gauge_coord(const float* Gcol, int gstride, const float* x, int g) {
+    if (g <= 16) {
+        float acc = 0.0f;
+        for (int j = 0; j < g; j++) acc = fmaf(Gcol[j * gstride], x[j], acc);
+        return acc;
+    }
+    const int nb = g >> 4;
+    float p[8];
+#pragma unroll
+    for (int b = 0; b < 8; b++) p[b] = 0.0f;
+#pragma unroll 4
+    for (int jj = 0; jj < 16; jj++) {
+#pragma unroll
+        for (int b = 0; b < 8; b++)
+            if (b < nb) p[b] = fmaf(Gcol[(16 * b + jj) * gstride], x[16 * b + jj], p[b]);
+    }
+    float acc = p[0];
+#pragma unroll
+    for (int b = 1; b < 8; b++)
+        if (b < nb) acc = __fadd_rn(acc, p[b]);
+    return acc;
 }
 
 // Extract the b-bit code that starts at bit p of a little-endian word stream.
@@ -97,11 +123,7 @@ __global__ void __launch_bounds__(kRowThreads) row_encode_kernel(RowArgs a) {
 #pragma unroll
         for (int k = 0; k < NR; k++) {
             const int c = lane + 32 * k, r = c / g, i = c - r * g;
-            const float* Gcol = Gs + r * g * g + i;
-            const float* xg = xs + r * g;
-            float acc = 0.0f;
-            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], xg[jj], acc);
-            z[k] = acc;
+            z[k] = gauge_coord(Gs + r * g * g + i, g, xs + r * g, g);
         }
         const int64_t coff = a.cmap.at(l, s, b, h, t);
         if (a.none_mode) {
@@ -208,10 +230,7 @@ __global__ void __launch_bounds__(kRowThreads) row_decode_kernel(RowArgs a) {
 #pragma unroll
         for (int k = 0; k < NR; k++) {
             const int c = lane + 32 * k, r = c / g, i = c - r * g;
-            const float* Gcol = Gs + r * g * g + i;
-            const float* zg = zs + r * g;
-            float acc = 0.0f;
-            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], zg[jj], acc);
+            const float acc = gauge_coord(Gs + r * g * g + i, g, zs + r * g, g);
             orow[c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
         }
         __syncwarp();
@@ -256,11 +275,7 @@ __global__ void __launch_bounds__(kRowThreads) key_encode_kernel(KeyArgs a) {
 #pragma unroll
         for (int k = 0; k < NR; k++) {
             const int c = lane + 32 * k, r = c / g, i = c - r * g;
-            const float* Gcol = Gs + r * g * g + i;
-            const float* xg = xs + r * g;
-            float acc = 0.0f;
-            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], xg[jj], acc);
-            Zs[(size_t)t * d + c] = acc;
+            Zs[(size_t)t * d + c] = gauge_coord(Gs + r * g * g + i, g, xs + r * g, g);
         }
         __syncwarp();
     }
@@ -340,10 +355,7 @@ __global__ void __launch_bounds__(kRowThreads) key_decode_kernel(KeyArgs a) {
 #pragma unroll
         for (int k = 0; k < NR; k++) {
             const int c = lane + 32 * k, r = c / g, i = c - r * g;
-            const float* Gcol = Gs + r * g * g + i;
-            const float* zg = zr + r * g;
-            float acc = 0.0f;
-            for (int jj = 0; jj < g; jj++) acc = fmaf(Gcol[jj * g], zg[jj], acc);
+            const float acc = gauge_coord(Gs + r * g * g + i, g, zr + r * g, g);
             O[(int64_t)t * d + c] = __bfloat16_as_ushort(__float2bfloat16_rn(acc));
         }
     }
