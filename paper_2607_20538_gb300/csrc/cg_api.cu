@@ -275,7 +275,7 @@ int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf1
         a.s_n = 1;
         a.t_count = z.nq;
         kivi_value_maps(shape, z, &a.cmap, &a.smap);
-        e = launch_row_encode_simt(a, st);
+        e = tc_row_encode_eligible(a) ? tc_launch_row_encode(a, st) : launch_row_encode_simt(a, st);
         if (e != cudaSuccess) return cuda_fail(e, "KIVI value encode launch");
     }
     if (shape->T - z.nq > 0) {
@@ -339,7 +339,7 @@ int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes,
         a.s_n = 1;
         a.t_count = z.nq;
         kivi_value_maps(shape, z, &a.cmap, &a.smap);
-        e = launch_row_decode_simt(a, st);
+        e = tc_row_decode_eligible(a) ? tc_launch_row_decode(a, st) : launch_row_decode_simt(a, st);
         if (e != cudaSuccess) return cuda_fail(e, "KIVI value decode launch");
     }
     if (shape->T - z.nq > 0) {

@@ -1,0 +1,425 @@
+// cg_tc_dec.cu -- tensor-core decode of the row path (Sec. 3: Zhat = D(B_c), Xhat = G^T Zhat),
+// head dim d = 128, block-uniform rows and KIVI value rows.
+//
+// Persistent warp-specialized kernel, one CTA per SM, 10 warps:
+//   warp 0      bulk-copy producer: the packed codes of a 128-token tile are contiguous
+//               (rows of 16*bits bytes); one cp.async.bulk per tile into a 4-stage ring;
+//   warp 1      MMA issuer: D_k = A_k B^T on tcgen05, A = codes as bf16 (128 + q, exact),
+//               B = G^T of the gauge group split into two bf16 terms; one fp32
+//               accumulator per quantization sub-block k of a group (block < group gives
+//               two), double buffered in tensor memory;
+//   warps 2..5  unpackers, one token row each: codes -> bf16 A tile (128-byte swizzle);
+//               at a gauge change they also build B and the per-column sums c_k[i] =
+//               sum_{j in sub-block k} G[j][i] of the split;
+//   warps 6..9  epilogue, one token row (TMEM lane) each:
+//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i], bf16 store.
+// With the scale and zero of a block constant along the token, dequantization commutes
+// with the rotation, so the integer codes go through the tensor cores unscaled.
+#include <cuda_bf16.h>
+
+#include "cg_sm100.cuh"
+#include "cg_tc.h"
+#include "cg_tc_common.cuh"
+
+namespace cg {
+namespace {
+
+using namespace sm100;
+using tc::kD;
+using tc::kWaitLimitNs;
+
+constexpr int kThreads = 320;
+constexpr int kCStages = 4;
+constexpr int kCStageBytes = 128 * 128;  // up to 8-bit codes: 128 rows x 128 B
+constexpr int kATile = 128 * kD * 2;
+constexpr int kSegBufs = 4;
+
+struct DecSmem {
+    static constexpr uint32_t a_tiles = 0;                          // 2 x 32 KB
+    static constexpr uint32_t bsplit = a_tiles + 2 * kATile;        // 2 x (16 or 32 KB)
+    static constexpr uint32_t cstages = bsplit + 2 * 32768;         // 4 x 16 KB
+    static constexpr uint32_t csum = cstages + kCStages * kCStageBytes;  // [4][2][128] fp32
+    static constexpr uint32_t misc = csum + kSegBufs * 2 * kD * 4;
+    static constexpr uint32_t total = misc + 512;
+};
+
+struct DecMisc {
+    uint64_t cfull[kCStages], cempty[kCStages];
+    uint64_t afull[2], aempty[2];
+    uint64_t accfull[2], accempty[2];
+    uint64_t gready[kSegBufs];
+    uint64_t bfree;
+    uint32_t tmem_slot;
+    int abort_flag;
+};
+
+struct DecParams {
+    RowArgs a;
+    tc::Sched S;
+    int nsub;  // accumulators per gauge group: group / block when block < group, else 1
+};
+
+// codes of one row (128 codes, little-endian bit stream) -> 16 chunks of 8 bf16 (128 + q)
+template <int BITS>
+__device__ __forceinline__ void unpack_row(const uint32_t* w, uint4 (&out)[16]) {
+#pragma unroll
+    for (int c = 0; c < 16; c++) {
+        uint32_t o[4];
+#pragma unroll
+        for (int e = 0; e < 4; e++) {
+            uint32_t q[2];
+#pragma unroll
+            for (int h = 0; h < 2; h++) {
+                const int k = 8 * c + 2 * e + h;
+                const int p = k * BITS;
+                uint32_t v = w[p >> 5] >> (p & 31);
+                if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
+                q[h] = v & ((1u << BITS) - 1u);
+            }
+            if (BITS < 8) {
+                o[e] = 0x43004300u | q[0] | (q[1] << 16);
+            } else {
+                const __nv_bfloat162 b2 = __floats2bfloat162_rn((float)q[0], (float)q[1]);
+                o[e] = *reinterpret_cast<const uint32_t*>(&b2);
+            }
+        }
+        out[c] = make_uint4(o[0], o[1], o[2], o[3]);
+    }
+}
+
+template <int BITS>
+__global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams P) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const uint32_t base_u32 = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    unsigned char* sm = smem_raw + (base_u32 - smem_u32(smem_raw));
+    DecMisc* M = reinterpret_cast<DecMisc*>(sm + DecSmem::misc);
+    unsigned char* atiles = sm + DecSmem::a_tiles;
+    unsigned char* bsplit = sm + DecSmem::bsplit;
+    unsigned char* cst = sm + DecSmem::cstages;
+    float* csum = reinterpret_cast<float*>(sm + DecSmem::csum);
+
+    const RowArgs& a = P.a;
+    const tc::Sched& S = P.S;
+    const int g = a.g, blk = a.blk, nsub = P.nsub;
+    const int gb = g < 16 ? 16 : g;
+    const uint32_t bsz = (g == 128) ? 32768u : 16384u;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int kRowBytes = 16 * BITS;
+    constexpr float kOff = BITS < 8 ? 128.0f : 0.0f;
+
+    const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
+    const int64_t t_end = S.n_tiles * (blockIdx.x + 1) / gridDim.x;
+    const int my_tiles = (int)(t_end - t_begin);
+    const int64_t seg0 = my_tiles > 0 ? tc::tile_info(a, S, t_begin).seg : 0;
+    const uint32_t acc_cols = (uint32_t)nsub * 128u;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kCStages; i++) {
+            mbar_init(&M->cfull[i], 1);
+            mbar_init(&M->cempty[i], 4);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&M->afull[i], 4);
+            mbar_init(&M->aempty[i], 1);
+            mbar_init(&M->accfull[i], 1);
+            mbar_init(&M->accempty[i], 4);
+        }
+        for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 4);
+        mbar_init(&M->bfree, 1);
+        M->abort_flag = 0;
+        fence_barrier_init();
+    }
+    for (uint32_t i = threadIdx.x; i < 2u * bsz / 16u; i += kThreads)
+        reinterpret_cast<uint4*>(bsplit)[i] = make_uint4(0, 0, 0, 0);
+    if (warp == 1) {
+        tmem_alloc(&M->tmem_slot, 2 * acc_cols);
+        tmem_relinquish();
+        tc_fence_before();
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = M->tmem_slot;
+    volatile int* abort_flag = &M->abort_flag;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ codes producer
+        if (lane == 0 && my_tiles > 0) {
+            int issued = 0;
+            for (int i = 0; i < my_tiles; i++) {
+                const int st = i % kCStages;
+                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+                const uint32_t bytes = (uint32_t)ti.rows_valid * kRowBytes;
+                mbar_arrive_expect_tx(&M->cfull[st], bytes);
+                bulk_load(cst + st * kCStageBytes, a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0), bytes,
+                          &M->cfull[st]);
+                issued = i + 1;
+            }
+            if (*abort_flag) {
+                const int zero = 0;
+                const int from = issued > kCStages ? issued - kCStages : 0;
+                for (int i = from; i < issued; i++)
+                    mbar_wait(&M->cfull[i % kCStages], (i / kCStages) & 1, &zero, kWaitLimitNs);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && my_tiles > 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, gb);
+            int64_t cur = -1;
+            int committed = 0;
+            for (int i = 0; i < my_tiles; i++) {
+                const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+                const int64_t ls = ti.seg - seg0;
+                bool ok = true;
+                if (ti.seg != cur) {
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    cur = ti.seg;
+                }
+                const int ab = i & 1, buf = i & 1;
+                ok = ok && mbar_wait(&M->afull[ab], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                if (!ok) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a_base = smem_u32(atiles + ab * kATile);
+                const uint32_t d_base = tmem + buf * acc_cols;
+                for (int p = 0; p < 2; p++) {
+                    const uint32_t b_base = smem_u32(bsplit) + p * bsz;
+                    for (int r = 0; r < 128 / gb; r++) {
+                        for (int k = 0; k < nsub; k++) {
+                            const int kw = nsub > 1 ? blk : gb;           // K width of this sub-block
+                            const int kbeg = r * gb + k * (nsub > 1 ? blk : 0);
+                            for (int ks = 0; ks < kw / 16; ks++) {
+                                const int k0 = kbeg + ks * 16;
+                                const uint32_t a_addr = a_base + (k0 >> 6) * 16384 + (k0 & 63) * 2;
+                                const uint32_t b_addr =
+                                    b_base + (g == 128 ? (k0 >> 6) * 16384 : 0) + (r * gb) * 128 + (k0 & 63) * 2;
+                                mma_bf16(d_base + k * 128 + r * gb, sdesc_sw128(a_addr), sdesc_sw128(b_addr), idesc,
+                                         (p > 0 || ks > 0) ? 1u : 0u);
+                            }
+                        }
+                    }
+                }
+                mma_commit(&M->accfull[buf]);
+                mma_commit(&M->aempty[ab]);
+                const bool last_of_seg =
+                    (i + 1 == my_tiles) || tc::tile_info(a, S, t_begin + i + 1).seg != ti.seg;
+                if (last_of_seg) mma_commit(&M->bfree);
+                committed = i + 1;
+            }
+            if (*abort_flag && committed > 0) {
+                const int zero = 0;
+                const int i = committed - 1;
+                mbar_wait(&M->accfull[i & 1], (i >> 1) & 1, &zero, kWaitLimitNs);
+            }
+        }
+    } else if (warp < 6) {
+        // ------------------------------------------------------------ unpackers / gauge
+        const int uw = warp - 2;
+        const int row = uw * 32 + lane;
+        int64_t cur = -1;
+        int nconv = 0;
+        for (int i = 0; i < my_tiles; i++) {
+            const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+            if (ti.seg != cur) {
+                const int64_t ls = ti.seg - seg0;
+                if (nconv > 0) {
+                    // the MMAs of the previous gauge set must be done with B
+                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                    if (!__all_sync(0xffffffffu, ok)) {
+                        *abort_flag = 1;
+                        break;
+                    }
+                }
+                // B[n][k] = G_r[k - r g][n - r g]: thread `row` builds output channel n = row
+                const int n = row, r = n / g, i_in = n - r * g;
+                const float* Gc = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g + (int64_t)r * g * g + i_in;
+                float cs[2] = {0.0f, 0.0f};
+                for (int j = 0; j < g; j += 8) {
+                    uint32_t hi[4], lo[4];
+#pragma unroll
+                    for (int e = 0; e < 8; e += 2) {
+                        const float v0 = __ldg(Gc + (int64_t)(j + e) * g);
+                        const float v1 = __ldg(Gc + (int64_t)(j + e + 1) * g);
+                        const __nv_bfloat16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
+                        const __nv_bfloat16 l0 = __float2bfloat16_rn(v0 - __bfloat162float(h0));
+                        const __nv_bfloat16 l1 = __float2bfloat16_rn(v1 - __bfloat162float(h1));
+                        hi[e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+                        lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+                        const float t2 = (__bfloat162float(h0) + __bfloat162float(l0)) +
+                                         (__bfloat162float(h1) + __bfloat162float(l1));
+                        const int ksub = (nsub > 1 && j + e >= blk) ? 1 : 0;
+                        cs[ksub] += t2;
+                    }
+                    const int k = r * g + j;
+                    unsigned char* reg1 = bsplit + 1 * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
+                    unsigned char* reg0 = bsplit + 0 * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
+                    *reinterpret_cast<uint4*>(reg1 + sw128_offset(n, k & 63)) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                    *reinterpret_cast<uint4*>(reg0 + sw128_offset(n, k & 63)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                }
+                float* cb = csum + (ls & 3) * 2 * kD;
+                cb[n] = cs[0];
+                cb[kD + n] = cs[1];
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
+                cur = ti.seg;
+                nconv++;
+            }
+            const int st = i % kCStages, ab = i & 1;
+            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, kWaitLimitNs);
+            ok = ok && mbar_wait(&M->aempty[ab], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, ok)) {
+                *abort_flag = 1;
+                break;
+            }
+            const uint4* src = reinterpret_cast<const uint4*>(cst + st * kCStageBytes + row * kRowBytes);
+            uint32_t w[4 * BITS + 1];
+#pragma unroll
+            for (int q = 0; q < BITS; q++) {
+                const uint4 v = src[q];
+                w[4 * q] = v.x;
+                w[4 * q + 1] = v.y;
+                w[4 * q + 2] = v.z;
+                w[4 * q + 3] = v.w;
+            }
+            w[4 * BITS] = 0;
+            uint4 outc[16];
+            unpack_row<BITS>(w, outc);
+            unsigned char* at = atiles + ab * kATile;
+#pragma unroll
+            for (int c = 0; c < 16; c++)
+                *reinterpret_cast<uint4*>(at + (c >> 3) * 16384 + row * 128 + (((c & 7) ^ (row & 7)) << 4)) = outc[c];
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&M->afull[ab]);
+                mbar_arrive(&M->cempty[st]);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int ew = warp & 3;
+        const int row = ew * 32 + lane;
+        for (int i = 0; i < my_tiles; i++) {
+            const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+            const int64_t ls = ti.seg - seg0;
+            const int buf = i & 1;
+            bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, ok)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const bool valid = row < ti.rows_valid;
+            const int nbk = kD / blk;
+            uint32_t sz[4] = {0, 0, 0, 0};
+            if (valid) {
+                const uint32_t* sp = a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
+#pragma unroll
+                for (int bk = 0; bk < 4; bk++)
+                    if (bk < nbk) sz[bk] = sp[bk];
+            }
+            const float* cb = csum + (ls & 3) * 2 * kD;
+            const uint32_t tacc = tmem + ((uint32_t)(ew * 32) << 16) + buf * acc_cols;
+            uint4* orow = reinterpret_cast<uint4*>(a.out + (tc::dense_row(a, ti) + row) * kD);
+#pragma unroll
+            for (int c = 0; c < 4; c++) {
+                // chunk c: columns 32c..32c+31; gauge group r = 32c / g (g >= 32) or several (g < 32)
+                const int r = (c * 32) / g;
+                float sk[2], ak[2];
+#pragma unroll
+                for (int k = 0; k < 2; k++) {
+                    const int bk = nsub > 1 ? (r * g + k * blk) / blk : (c * 32) / blk;
+                    uint32_t v = 0;
+#pragma unroll
+                    for (int q = 0; q < 4; q++)
+                        if (q == bk) v = sz[q];
+                    const float s = __half2float(__ushort_as_half((unsigned short)(v & 0xffffu)));
+                    const float m = __half2float(__ushort_as_half((unsigned short)(v >> 16)));
+                    sk[k] = s;
+                    ak[k] = m - kOff * s;
+                }
+                uint32_t d0[32], d1[32];
+                tmem_ld32(tacc + c * 32, d0);
+                if (nsub > 1) tmem_ld32(tacc + 128 + c * 32, d1);
+                tmem_wait_ld();
+                uint32_t o[16];
+#pragma unroll
+                for (int e = 0; e < 32; e += 2) {
+                    float x2[2];
+#pragma unroll
+                    for (int hh = 0; hh < 2; hh++) {
+                        const int col = c * 32 + e + hh;
+                        float xv = fmaf(sk[0], __uint_as_float(d0[e + hh]), ak[0] * cb[col]);
+                        if (nsub > 1) xv = fmaf(sk[1], __uint_as_float(d1[e + hh]), fmaf(ak[1], cb[kD + col], xv));
+                        x2[hh] = xv;
+                    }
+                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(x2[0], x2[1]);
+                    o[e >> 1] = *reinterpret_cast<const uint32_t*>(&b2);
+                }
+                if (valid) {
+#pragma unroll
+                    for (int q = 0; q < 4; q++) orow[c * 4 + q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&M->accempty[buf]);
+        }
+    }
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) raise_flag(a.status, CG_FLAG_PIPE_TIMEOUT);
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, 2 * acc_cols);
+    }
+}
+
+template <int BITS>
+cudaError_t launch_dec(const DecParams& P, cudaStream_t st) {
+    const size_t smem = DecSmem::total + 1024;
+    cudaError_t e = cudaFuncSetAttribute(tc_decode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
+    tc_decode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(P);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool tc_row_decode_eligible(const RowArgs& a) {
+    if (a.d != kD || a.none_mode) return false;
+    if (!(a.blk == 32 || a.blk == 64 || a.blk == 128)) return false;
+    if (a.blk < a.g && a.g / a.blk > 2) return false;
+    if (a.t_count < 64) return false;
+    if ((reinterpret_cast<uintptr_t>(a.codes) & 15u) || (reinterpret_cast<uintptr_t>(a.out) & 15u)) return false;
+    return true;
+}
+
+cudaError_t tc_launch_row_decode(const RowArgs& a, cudaStream_t st) {
+    DecParams P;
+    P.a = a;
+    P.S = tc::make_sched(a);
+    P.nsub = a.blk < a.g ? a.g / a.blk : 1;
+    if (P.S.n_tiles == 0) return cudaSuccess;
+    switch (a.bits) {
+        case 2: return launch_dec<2>(P, st);
+        case 3: return launch_dec<3>(P, st);
+        case 4: return launch_dec<4>(P, st);
+        case 6: return launch_dec<6>(P, st);
+        case 8: return launch_dec<8>(P, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace cg
