@@ -1,91 +1,113 @@
-// cg_tc.cu -- tensor-core (tcgen05) kernels of the row path, head dim d = 128.
+// cg_tc.cu -- tensor-core (tcgen05) encode of the row path, head dim d = 128: gauge
+// rotation (Sec. 3, Z = G X) fused with the block-uniform quantizer of Sec. 4.3 (one range
+// per block of `block` channels of a token), also used for KIVI value rows.
 //
-// Encode (Sec. 3: Z = G X, then the block-uniform backend of Sec. 4.3) as one persistent,
-// warp-specialized kernel per launch:
-//   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte swizzle)
-//               into a ring of kStages shared-memory stages;
-//   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group, one
-//               MMA chain per group block), with G split into npass bf16 terms (hi + lo
-//               [+ lo2]) so that z~ is within a few fp32 ulps of the exact product; fp32
-//               accumulators in tensor memory, double buffered;
-//   warps 2..5  epilogue, one thread per token row (= TMEM lane): block min/max, fp16
-//               scale/zero, codes, bit packing, stores.
-// Exactness: the library defines z as a fixed-order fp32 sum (16-wide fma chains; see
-// include/codecgauge.h). z~ differs from it by at most E = ||x_group||_2 * e_i, with e_i
-// built per gauge row from the rounding bound of that order, the measured error model of
-// the tensor-core accumulation and the exact residual of the bf16 split. The epilogue
-// decides the fp16 scale/zero from the interval [z~ - E, z~ + E] when every value in it
-// rounds to the same fp16 result; otherwise it recomputes the candidate extremes exactly.
-// Codes whose pre-rounding value lies within E/s of a rounding boundary are recomputed
-// exactly too. Recomputation uses the same fixed-order sum as the CUDA-core kernels,
-// spread over the lanes of a warp through a small shared-memory job queue.
+// Persistent warp-specialized kernel, one CTA per SM, 11 warps:
+//   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte
+//               swizzle) into a 4-stage ring;
+//   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group,
+//               one MMA chain per group block), G split into npass bf16 terms (hi + lo
+//               [+ lo2]); fp32 accumulators in tensor memory, two buffers;
+//   warp 2      gauge converter: at each gauge change builds the bf16 split operand and
+//               the per-block error coefficients of the new gauge set;
+//   warps 3..10 two epilogue warpgroups; warpgroup k owns accumulator buffer k and takes
+//               every other tile; one thread per token row (= TMEM lane): block min/max,
+//               fp16 scale/zero, codes, packing, stores.
+//
+// Exactness. The library defines z as a fixed-order fp32 sum (16-wide fma chains, slice
+// sums added left to right; include/codecgauge.h). For every output channel i the
+// converter bounds |z~_i - z_i| / ||x_group||_2 by
+//     e_i = (c_order + c_tc) ||G_i||_2 + ||G_i - sum of split terms||_2,
+// c_order the rounding bound of the fixed order, c_tc a bound on the tensor-core fp32
+// accumulation (measured well below it), and the exact residual of the bf16 split. The
+// epilogue turns it into E per block. A block's fp16 scale and zero are monotone functions
+// of its (max, min); when every (max, min) within E of the approximate ones gives the same
+// fp16 results they are taken directly, otherwise the candidate extremes are recomputed
+// exactly. A code is taken from z~ unless its pre-rounding value lies within E/s of a
+// rounding boundary; those are recomputed exactly. Recomputation uses the library's order
+// (as the CUDA-core kernels do), spread over the lanes of a warp by a shared-memory job
+// queue, so codes, scales and zeros are bit-identical to the definition.
 #include <cuda_bf16.h>
-
-#include <cstdio>
-#include <mutex>
 
 #include "cg_sm100.cuh"
 #include "cg_tc.h"
+#include "cg_tc_common.cuh"
 #include "cg_tmap.h"
 
 namespace cg {
 namespace {
 
 using namespace sm100;
+using tc::kD;
+using tc::kWaitLimitNs;
 
-constexpr int kD = 128;                 // head dimension handled here
-constexpr int kStages = 4;              // x tile ring
+constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
-constexpr int kThreads = 192;
-constexpr int kQCap = 96;               // repair jobs per warp and round
-constexpr uint64_t kWaitLimitNs = 4000000000ull;
-constexpr float kU = 5.9604645e-08f;    // 2^-24
+constexpr int kThreads = 352;
+constexpr int kEpiWarp0 = 3;
+constexpr int kQCap = 64;             // repair jobs per warp and round
+constexpr int kSegBufs = 4;
+constexpr float kU = 5.9604645e-08f;  // 2^-24
+constexpr float kMagic = 12582912.0f; // 1.5 * 2^23: adding it rounds to an integer (RNE)
 
 struct EncSmem {
-    // byte offsets from the 1024-aligned base
     static constexpr uint32_t stages = 0;
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // npass x (16 or 32 KB)
-    static constexpr uint32_t bsplit_max = 3 * 16384 > 2 * 32768 ? 3 * 16384 : 2 * 32768;
-    static constexpr uint32_t codes_stage = bsplit + bsplit_max;       // 128 rows x (4*BITS+4) words
-    static constexpr uint32_t codes_stage_max = 128 * (4 * 8 + 4) * 4;
-    static constexpr uint32_t queue = codes_stage + codes_stage_max;   // 4 warps x kQCap x 8 B
-    static constexpr uint32_t misc = queue + 4 * kQCap * 8;
-    static constexpr uint32_t total = misc + 1024;
+    static constexpr uint32_t queue = bsplit + 65536;                  // 8 warps x kQCap x 8 B
+    static constexpr uint32_t misc = queue + 8 * kQCap * 8;
+    static constexpr uint32_t total = misc + 512;
 };
 
 struct Misc {
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t acc_full[2];
-    uint64_t acc_empty[2];
-    uint64_t g_ready;
+    uint64_t full[kStages], empty[kStages];
+    uint64_t accfull[2], accempty[2];
+    uint64_t gready[kSegBufs];
+    uint64_t bfree;
     uint32_t tmem_slot;
     int abort_flag;
-    int qcount[4];
-    float emax[2][4][16];  // [conversion parity][epilogue warp][gauge group]: max_i e_i
+    int qcount[8];
+    float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
 };
 
 struct EncParams {
     RowArgs a;
+    tc::Sched S;
     int npass;
-    int64_t n_units, tiles_per_unit, n_tiles;
 };
 
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
-// unit index (b fastest, then h, s, l) -> (l, s, b, h); tiles of a unit are contiguous
-__device__ __forceinline__ void unit_coords(const RowArgs& a, int64_t u, int& l, int& s, int& b, int& h) {
-    b = (int)(u % a.B);
-    int64_t r = u / a.B;
-    h = (int)(r % a.H);
-    r /= a.H;
-    s = a.s_lo + (int)(r % a.s_n);
-    l = (int)(r / a.s_n);
+__device__ __forceinline__ float min3f(float a, float b, float c) {
+    float r;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+template <typename T>
+__device__ __forceinline__ T pick4(const T (&v)[4], int i) {
+    return i == 0 ? v[0] : i == 1 ? v[1] : i == 2 ? v[2] : v[3];
+}
+
+// Rows of the gauge channels whose error bounds block bk's values: the whole gauge group
+// when the group spans the block, else the block's own channels.
+__device__ __forceinline__ void bound_range(int bk, int g, int blk, int& lo, int& hi) {
+    if (g >= blk) {
+        lo = ((bk * blk) / g) * g;
+        hi = lo + g;
+    } else {
+        lo = bk * blk;
+        hi = lo + blk;
+    }
 }
 
 // Exact gauge-space value of (row, col) in the library's fixed order, x read from the
-// swizzled stage tile and G from global memory (fp32, row `col` of the head's gauge set).
+// swizzled stage tile and G from global memory (fp32 row `col` of the head's gauge set).
 __device__ __noinline__ float exact_z(const unsigned char* stage, int row, int col, const float* Gf, int g) {
     const int r0 = (col / g) * g;
     const float* Grow = Gf + (size_t)col * g;
@@ -123,9 +145,24 @@ __device__ __noinline__ float exact_z(const unsigned char* stage, int row, int c
     return acc;
 }
 
-// fp16 scale of a block with the given (max, min) in fp32, by the library's rule.
 __device__ __forceinline__ uint32_t scale16(float mx, float mn, float qmax) {
     return f2h_bits(__fdiv_rn(__fsub_rn(mx, mn), qmax));
+}
+
+// Overwrite the BITS-bit code at bit position `bit` of a packed row in global memory
+// (the row was stored by this thread; the rare exact recomputes are patched in place).
+template <int BITS>
+__device__ __forceinline__ void patch_code(uint8_t* rowp, int bit, uint32_t q) {
+    unsigned int* wp = reinterpret_cast<unsigned int*>(rowp) + (bit >> 5);
+    const int off = bit & 31;
+    const uint32_t msk = (1u << BITS) - 1u;
+    atomicAnd(wp, ~(msk << off));
+    atomicOr(wp, q << off);
+    if (off + BITS > 32) {
+        const int sh = 32 - off;
+        atomicAnd(wp + 1, ~(msk >> sh));
+        atomicOr(wp + 1, q >> sh);
+    }
 }
 
 template <int BITS>
@@ -137,19 +174,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     Misc* M = reinterpret_cast<Misc*>(sm + EncSmem::misc);
     unsigned char* stages = sm + EncSmem::stages;
     unsigned char* bsplit = sm + EncSmem::bsplit;
-    uint32_t* cstage = reinterpret_cast<uint32_t*>(sm + EncSmem::codes_stage);
     uint32_t* queue = reinterpret_cast<uint32_t*>(sm + EncSmem::queue);
 
     const RowArgs& a = P.a;
+    const tc::Sched& S = P.S;
     const int g = a.g, blk = a.blk, npass = P.npass;
     const int gb = g < 16 ? 16 : g;
+    const int nbk = kD / blk;
     const uint32_t bsz = (g == 128) ? 32768u : 16384u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // contiguous tile range of this CTA
-    const int64_t t_begin = P.n_tiles * blockIdx.x / gridDim.x;
-    const int64_t t_end = P.n_tiles * (blockIdx.x + 1) / gridDim.x;
+    const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
+    const int64_t t_end = S.n_tiles * (blockIdx.x + 1) / gridDim.x;
     const int my_tiles = (int)(t_end - t_begin);
+    const int64_t seg0 = my_tiles > 0 ? tc::tile_info(a, S, t_begin).seg : 0;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kStages; i++) {
@@ -157,15 +195,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             mbar_init(&M->empty[i], 4);
         }
         for (int i = 0; i < 2; i++) {
-            mbar_init(&M->acc_full[i], 1);
-            mbar_init(&M->acc_empty[i], 4);
+            mbar_init(&M->accfull[i], 1);
+            mbar_init(&M->accempty[i], 4);
         }
-        mbar_init(&M->g_ready, 4);
+        for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 1);
+        mbar_init(&M->bfree, 1);
         M->abort_flag = 0;
-        for (int i = 0; i < 4; i++) M->qcount[i] = 0;
         fence_barrier_init();
     }
-    // zero the B operand area once: off-diagonal gauge blocks stay zero
     for (uint32_t i = threadIdx.x; i < (uint32_t)npass * bsz / 16; i += kThreads)
         reinterpret_cast<uint4*>(bsplit)[i] = make_uint4(0, 0, 0, 0);
     if (warp == 1) {
@@ -184,18 +221,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         if (lane == 0 && my_tiles > 0) {
             prefetch_tmap(&xmap);
             int issued = 0;
-            for (int i = 0; i < my_tiles; i++) {
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
                 const int st = i % kStages;
                 if (!mbar_wait(&M->empty[st], ((i / kStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     *abort_flag = 1;
                     break;
                 }
-                const int64_t tile = t_begin + i;
-                const int64_t u = tile / P.tiles_per_unit;
-                const int64_t t0 = (tile - u * P.tiles_per_unit) * 128;
-                int l, s, b, h;
-                unit_coords(a, u, l, s, b, h);
-                const int64_t row0 = (((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t0;
+                const tc::TileInfo ti = it.info(a);
+                const int64_t row0 = tc::dense_row(a, ti);
                 unsigned char* dst = stages + st * kTileBytes;
                 mbar_arrive_expect_tx(&M->full[st], kTileBytes);
                 tma_load_2d(dst, &xmap, &M->full[st], 0, (int)row0);
@@ -203,9 +238,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 issued = i + 1;
             }
             if (*abort_flag) {
-                // let every load this thread issued land before the CTA can exit
-                const int from = issued > kStages ? issued - kStages : 0;
                 const int zero = 0;
+                const int from = issued > kStages ? issued - kStages : 0;
                 for (int i = from; i < issued; i++)
                     mbar_wait(&M->full[i % kStages], (i / kStages) & 1, &zero, kWaitLimitNs);
             }
@@ -214,24 +248,21 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && my_tiles > 0) {
             const uint32_t idesc = idesc_bf16_f32(128, gb);
-            int64_t cur_gid = -1;
-            int g_phase = 0;
+            int64_t cur = -1;
             int committed = 0;
-            for (int i = 0; i < my_tiles; i++) {
-                const int64_t tile = t_begin + i;
-                const int64_t u = tile / P.tiles_per_unit;
-                int l, s, b, h;
-                unit_coords(a, u, l, s, b, h);
-                const int64_t gid = (int64_t)(l * 2 + s) * a.H + h;
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+                const tc::TileInfo ti = it.info(a);
+                const int64_t ls = ti.seg - seg0;
                 bool ok = true;
-                if (gid != cur_gid) {
-                    ok = mbar_wait(&M->g_ready, g_phase, abort_flag, kWaitLimitNs);
-                    g_phase ^= 1;
-                    cur_gid = gid;
+                if (ti.seg != cur) {
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    cur = ti.seg;
                 }
                 const int st = i % kStages, buf = i & 1;
                 ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
-                ok = ok && mbar_wait(&M->acc_empty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
                 if (!ok) {
                     *abort_flag = 1;
                     break;
@@ -252,50 +283,42 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         }
                     }
                 }
-                mma_commit(&M->acc_full[buf]);
+                mma_commit(&M->accfull[buf]);
+                const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
+                if (last_of_seg) mma_commit(&M->bfree);
                 committed = i + 1;
             }
             if (*abort_flag && committed > 0) {
                 const int zero = 0;
                 const int i = committed - 1;
-                mbar_wait(&M->acc_full[i & 1], (i >> 1) & 1, &zero, kWaitLimitNs);
+                mbar_wait(&M->accfull[i & 1], (i >> 1) & 1, &zero, kWaitLimitNs);
             }
         }
-    } else {
-        // ------------------------------------------------------------ epilogue
-        const int ew = warp & 3;              // TMEM lane quadrant of this warp
-        const int row = ew * 32 + lane;       // tile row = TMEM lane
-        const int etid = (warp - 2) * 32 + lane;  // B row this thread converts
-        const int qw = warp - 2;
-        uint32_t* qjob = queue + qw * kQCap * 2;       // (row | col << 8), result bits
-        const int R = kD / g;
-        const int nbk = kD / blk;
-        const float qmaxf = (float)((1 << BITS) - 1);
-        const int qmax = (1 << BITS) - 1;
-        constexpr int kWords = 4 * BITS;               // packed words per row (128 codes)
-        constexpr int kStride = kWords + 4;
-        uint32_t* my_codes = cstage + row * kStride;
-        // error coefficients of the fixed-order sum and of the tensor-core accumulation
+    } else if (warp == 2) {
+        // ------------------------------------------------------------ gauge converter
         const int n_order = (g < 16 ? g : 16) + (g >= 16 ? g / 16 : 1) - 1;
-        const float c_chain = (float)n_order * kU * 1.01f;
+        const float c_order = (float)n_order * kU * 1.01f;
         const float c_tc = 2.0f * (float)(npass * (gb / 16) + 2) * kU;
-        int32_t flag = 0;
-        int64_t cur_gid = -1;
-        int conv = 0;  // gauge conversions done by this warp
-        const float* Gf = nullptr;
-        bool ok = true;
-
-        for (int i = 0; i < my_tiles && ok; i++) {
-            const int64_t tile = t_begin + i;
-            const int64_t u = tile / P.tiles_per_unit;
-            const int64_t t0 = (tile - u * P.tiles_per_unit) * 128;
-            int l, s, b, h;
-            unit_coords(a, u, l, s, b, h);
-            const int64_t gid = (int64_t)(l * 2 + s) * a.H + h;
-            if (gid != cur_gid) {
-                // ---- convert the gauge set of (l, s, h) into the bf16 split operand
-                Gf = a.G + gid * (int64_t)kD * g;
-                const int n = etid;  // B row = output channel
+        int64_t cur = -1;
+        int nconv = 0;
+        tc::TileIter it;
+        it.init(a, S, t_begin);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            const tc::TileInfo ti = it.info(a);
+            if (ti.seg == cur) continue;
+            const int64_t ls = ti.seg - seg0;
+            if (nconv > 0) {
+                const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                if (!__all_sync(0xffffffffu, ok)) {
+                    *abort_flag = 1;
+                    break;
+                }
+            }
+            const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
+            float e_row[4];
+#pragma unroll
+            for (int q = 0; q < 4; q++) {
+                const int n = lane + 32 * q;  // B row = output channel
                 const int r = n / g;
                 const float* Gr = Gf + (size_t)n * g;
                 float s_g2 = 0.0f, s_res2 = 0.0f;
@@ -304,7 +327,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     const float4 v0 = __ldg(reinterpret_cast<const float4*>(Gr + j));
                     const float4 v1 = __ldg(reinterpret_cast<const float4*>(Gr + j + 4));
                     const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
-                    // term t = 0 is the leading bf16 part; pass p uses term npass - 1 - p
                     uint32_t term[3][4];
 #pragma unroll
                     for (int e = 0; e < 8; e += 2) {
@@ -328,132 +350,141 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 #pragma unroll
                     for (int t = 0; t < 3; t++) {
                         if (t < npass) {
-                            const int pp = npass - 1 - t;
-                            unsigned char* region = bsplit + pp * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
+                            unsigned char* region = bsplit + (npass - 1 - t) * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
                             *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
                                 make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
                         }
                     }
                 }
-                // e_n bounds |z~ - z| / ||x_group||_2 for this output channel; each warp keeps
-                // the maximum over the rows of each group it covers
-                float e_n = ((c_chain + c_tc) * sqrtf(s_g2) + sqrtf(s_res2)) * 1.001f + 1e-30f;
-                const int seg = g < 32 ? g : 32;
-                for (int off = seg >> 1; off >= 1; off >>= 1) e_n = fmaxf(e_n, __shfl_xor_sync(0xffffffffu, e_n, off));
-                if ((lane & (seg - 1)) == 0) M->emax[conv & 1][qw][r] = e_n;
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&M->g_ready);
-                // every epilogue warp's part (B operand and bounds) is written once the phase completes
-                const bool g_ok = mbar_wait(&M->g_ready, conv & 1, abort_flag, kWaitLimitNs);
-                if (!__all_sync(0xffffffffu, g_ok)) {
-                    *abort_flag = 1;
-                    ok = false;
-                    break;
-                }
-                cur_gid = gid;
-                conv++;
+                e_row[q] = ((c_order + c_tc) * sqrtf(s_g2) + sqrtf(s_res2)) * 1.001f + 1e-30f;
             }
-            const int st = i % kStages, buf = i & 1;
-            // accumulator ready; the stage's TMA data is acquired through its own barrier
-            // (already complete: this warp releases the stage only after the tile)
-            bool w_ok = mbar_wait(&M->acc_full[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
-            w_ok = w_ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
-            if (!__all_sync(0xffffffffu, w_ok)) {
+            // per quantization block: max of e over the rows that bound its values
+#pragma unroll
+            for (int bk = 0; bk < 4; bk++) {
+                if (bk < nbk) {
+                    int lo, hi;
+                    bound_range(bk, g, blk, lo, hi);
+                    float m = 0.0f;
+#pragma unroll
+                    for (int q = 0; q < 4; q++) {
+                        const int n = lane + 32 * q;
+                        if (n >= lo && n < hi) m = fmaxf(m, e_row[q]);
+                    }
+                    for (int off = 16; off >= 1; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+                    if (lane == 0) M->emaxb[ls & 3][bk] = m;
+                }
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
+            cur = ti.seg;
+            nconv++;
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue warpgroups
+        const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup = accumulator buffer
+        const int q4 = warp & 3;                      // TMEM lane quadrant of this warp
+        const int row = q4 * 32 + lane;               // tile row = TMEM lane
+        const int qw = warp - kEpiWarp0;              // job queue of this warp
+        uint32_t* qjob = queue + qw * kQCap * 2;
+        const float qmaxf = (float)((1 << BITS) - 1);
+        const int qmax = (1 << BITS) - 1;
+        int lo8[4], hi8[4];
+#pragma unroll
+        for (int bk = 0; bk < 4; bk++) {
+            int lo = 0, hi = 0;
+            if (bk < nbk) bound_range(bk, g, blk, lo, hi);
+            lo8[bk] = lo >> 3;
+            hi8[bk] = hi >> 3;
+        }
+        int32_t flag = 0;
+        tc::TileIter it;
+        it.init(a, S, t_begin + wg);
+        for (int i = wg; i < my_tiles; i += 2, it.step(a, 2)) {
+            const tc::TileInfo ti = it.info(a);
+            const int64_t ls = ti.seg - seg0;
+            const int st = i % kStages, buf = wg;
+            bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+            ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
+            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
-                ok = false;
                 break;
             }
             tc_fence_after();
             const unsigned char* stg = stages + st * kTileBytes;
-            const int rows_valid = (int)((a.t_count - t0) < 128 ? (a.t_count - t0) : 128);
-            const bool valid = row < rows_valid;
-            const uint32_t tacc = tmem + ((uint32_t)(ew * 32) << 16) + buf * 128;
+            const bool valid = row < ti.rows_valid;
+            const uint32_t tacc = tmem + ((uint32_t)(q4 * 32) << 16) + buf * 128;
+            const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
 
-            // ---- 1. per-group norms of x from the stage (bf16 exact -> fp32)
-            float nrm2[16];
+            // ---- 1. ||x||^2 over the bound range of every block (bf16 -> fp32 exact)
+            float bs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-            for (int r = 0; r < 16; r++) nrm2[r] = 0.0f;
-            bool nonfinite = false;
+            for (int c8 = 0; c8 < 16; c8++) {
+                const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
+                                                                 (((c8 & 7) ^ (row & 7)) << 4));
+                float s0 = bf_lo(xv.x) * bf_lo(xv.x);
+                s0 = fmaf(bf_hi(xv.x), bf_hi(xv.x), s0);
+                s0 = fmaf(bf_lo(xv.y), bf_lo(xv.y), s0);
+                s0 = fmaf(bf_hi(xv.y), bf_hi(xv.y), s0);
+                s0 = fmaf(bf_lo(xv.z), bf_lo(xv.z), s0);
+                s0 = fmaf(bf_hi(xv.z), bf_hi(xv.z), s0);
+                s0 = fmaf(bf_lo(xv.w), bf_lo(xv.w), s0);
+                s0 = fmaf(bf_hi(xv.w), bf_hi(xv.w), s0);
 #pragma unroll
-            for (int c = 0; c < 16; c++) {
-                const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c >> 3) * 16384 + row * 128 +
-                                                                 (((c & 7) ^ (row & 7)) << 4));
-                const uint32_t wv[4] = {xv.x, xv.y, xv.z, xv.w};
-                float acc = 0.0f;
-#pragma unroll
-                for (int q = 0; q < 4; q++) {
-                    const float lo = bf_lo(wv[q]), hi = bf_hi(wv[q]);
-                    acc = fmaf(lo, lo, acc);
-                    acc = fmaf(hi, hi, acc);
-                    nonfinite |= ((wv[q] >> 7) & 0xffu) == 0xffu || ((wv[q] >> 23) & 0xffu) == 0xffu;
+                for (int bk = 0; bk < 4; bk++)
+                    if (c8 >= lo8[bk] && c8 < hi8[bk]) bs[bk] += s0;
+            }
+            if (valid && !(isfinite(bs[0]) && isfinite(bs[1]) && isfinite(bs[2]) && isfinite(bs[3]))) {
+                // a non-finite sum of squares: look for an Inf/NaN input (huge finite values
+                // can also overflow the square)
+                for (int c8 = 0; c8 < 16; c8++) {
+                    const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
+                                                                     (((c8 & 7) ^ (row & 7)) << 4));
+                    const uint32_t wv[4] = {xv.x, xv.y, xv.z, xv.w};
+                    for (int q = 0; q < 4; q++)
+                        if (bf16_nonfinite(wv[q] & 0xffffu) || bf16_nonfinite(wv[q] >> 16)) flag |= CG_FLAG_NONFINITE_INPUT;
                 }
-                // chunk c holds channels 8c..8c+7, inside group (8c)/g
-#pragma unroll
-                for (int r = 0; r < 16; r++)
-                    if (r == (8 * c) / g) nrm2[r] += acc;
             }
-            if (valid && nonfinite) flag |= CG_FLAG_NONFINITE_INPUT;
 
-            // ---- 2. approximate block ranges and their error bound
-            float mnv[4], mxv[4], Eb[4];
-#pragma unroll
-            for (int bk = 0; bk < 4; bk++) {
-                mnv[bk] = INFINITY;
-                mxv[bk] = -INFINITY;
-                Eb[bk] = 0.0f;
-            }
-#pragma unroll
+            // ---- 2. approximate block ranges from the accumulator
+            float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+            float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             for (int c = 0; c < 4; c++) {
                 uint32_t v[32];
                 tmem_ld32(tacc + c * 32, v);
                 tmem_wait_ld();
-                const int bk = (c * 32) / blk;
                 float lo = __uint_as_float(v[0]), hi = lo;
 #pragma unroll
-                for (int k = 1; k < 32; k++) {
-                    lo = fminf(lo, __uint_as_float(v[k]));
-                    hi = fmaxf(hi, __uint_as_float(v[k]));
+                for (int k = 1; k < 31; k += 2) {
+                    lo = min3f(lo, __uint_as_float(v[k]), __uint_as_float(v[k + 1]));
+                    hi = max3f(hi, __uint_as_float(v[k]), __uint_as_float(v[k + 1]));
                 }
+                lo = fminf(lo, __uint_as_float(v[31]));
+                hi = fmaxf(hi, __uint_as_float(v[31]));
+                const int bk = (c * 32) / blk;
 #pragma unroll
                 for (int q = 0; q < 4; q++)
                     if (q == bk) {
-                        mnv[q] = fminf(mnv[q], lo);
-                        mxv[q] = fmaxf(mxv[q], hi);
+                        mn[q] = fminf(mn[q], lo);
+                        mx[q] = fmaxf(mx[q], hi);
                     }
-            }
-            // E per block: max over the gauge groups it overlaps (group bound = ||x_r|| * max_w emax)
-            {
-                const float (*em)[16] = M->emax[(conv - 1) & 1];
-#pragma unroll
-                for (int r = 0; r < 16; r++) {
-                    if (r < R) {
-                        float e = 0.0f;
-                        // warps whose 32 rows intersect group r
-                        const int w0 = (r * g) >> 5, w1 = ((r + 1) * g - 1) >> 5;
-                        for (int w = w0; w <= w1; w++) e = fmaxf(e, em[w][r]);
-                        const float er = sqrtf(nrm2[r]) * 1.0001f * e;
-#pragma unroll
-                        for (int bk = 0; bk < 4; bk++)
-                            if (bk < nbk && r * g < (bk + 1) * blk && (r + 1) * g > bk * blk) Eb[bk] = fmaxf(Eb[bk], er);
-                    }
-                }
-#pragma unroll
-                for (int bk = 0; bk < 4; bk++) Eb[bk] += (fabsf(mnv[bk]) + fabsf(mxv[bk])) * 2.4e-7f;
             }
 
-            // ---- 3. decide scale/zero from the intervals; flag ambiguous blocks
+            // ---- 3. error bound per block; scale/zero from the intervals when they agree
+            float E[4];
             uint32_t s16[4], m16[4];
-            int amb = 0;  // bit 2*bk: scale ambiguous, bit 2*bk+1: zero ambiguous
+            int amb = 0;  // bit 2bk: scale needs the exact extremes; bit 2bk+1: zero needs the exact min
 #pragma unroll
             for (int bk = 0; bk < 4; bk++) {
+                E[bk] = 0.0f;
                 s16[bk] = m16[bk] = 0;
                 if (bk < nbk) {
-                    const float E = Eb[bk];
-                    const float mn_lo = __fsub_rn(mnv[bk], E), mn_hi = __fadd_rn(mnv[bk], E);
-                    const float mx_lo = __fsub_rn(mxv[bk], E), mx_hi = __fadd_rn(mxv[bk], E);
-                    const float dlo = fmaxf(__fsub_rn(mx_lo, mn_hi), 0.0f);
-                    const uint32_t slo = f2h_bits(__fdiv_rn(dlo, qmaxf));
+                    E[bk] = sqrtf(bs[bk]) * 1.0001f * M->emaxb[ls & 3][bk] + (fabsf(mn[bk]) + fabsf(mx[bk])) * 2.4e-7f;
+                    const float e = E[bk];
+                    const float mn_lo = __fsub_rn(mn[bk], e), mn_hi = __fadd_rn(mn[bk], e);
+                    const float mx_lo = __fsub_rn(mx[bk], e), mx_hi = __fadd_rn(mx[bk], e);
+                    const uint32_t slo = f2h_bits(__fdiv_rn(fmaxf(__fsub_rn(mx_lo, mn_hi), 0.0f), qmaxf));
                     const uint32_t shi = scale16(mx_hi, mn_lo, qmaxf);
                     const uint32_t mlo = f2h_bits(mn_lo), mhi = f2h_bits(mn_hi);
                     s16[bk] = slo;
@@ -462,66 +493,58 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     if (valid && mlo != mhi) amb |= 2 << (2 * bk);
                 }
             }
-            // ---- 4. exact recompute of the candidate extremes of ambiguous blocks
-            float ex_mn[4], ex_mx[4];
-#pragma unroll
-            for (int bk = 0; bk < 4; bk++) {
-                ex_mn[bk] = INFINITY;
-                ex_mx[bk] = -INFINITY;
-            }
-            int myslot[8], mytag[8];
-            int nmine = 0;
+
+            // ---- 4. exact extremes of ambiguous blocks (warp-cooperative)
             if (__any_sync(0xffffffffu, amb != 0)) {
+                float ex_mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+                float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                int nmine = 0;
+                int ms[4] = {0, 0, 0, 0}, mt[4] = {0, 0, 0, 0};
                 if (lane == 0) M->qcount[qw] = 0;
                 __syncwarp();
-#pragma unroll
                 for (int c = 0; c < 4; c++) {
                     const int bk = (c * 32) / blk;
-                    const int need = (amb >> (2 * bk)) & 3;  // any side ambiguous -> need min; scale -> max too
+                    const int need = (amb >> (2 * bk)) & 3;
                     if (!__any_sync(0xffffffffu, need != 0)) continue;
                     uint32_t v[32];
                     tmem_ld32(tacc + c * 32, v);
                     tmem_wait_ld();
-                    if (need) {
-                        float E = 0.0f, mnb = 0.0f, mxb = 0.0f;
+                    if (!need) continue;
+                    const float e = pick4(E, bk);
+                    const float thr_lo = __fadd_rn(pick4(mn, bk), 2.0f * e);
+                    const float thr_hi = __fsub_rn(pick4(mx, bk), 2.0f * e);
+                    uint32_t mmin = 0, mmax = 0;
 #pragma unroll
-                        for (int q = 0; q < 4; q++)
-                            if (q == bk) {
-                                E = Eb[q];
-                                mnb = mnv[q];
-                                mxb = mxv[q];
-                            }
-                        const float thr_lo = __fadd_rn(mnb, 2.0f * E), thr_hi = __fsub_rn(mxb, 2.0f * E);
-                        uint32_t mmin = 0, mmax = 0;
+                    for (int k = 0; k < 32; k++) {
+                        const float z = __uint_as_float(v[k]);
+                        if (z <= thr_lo) mmin |= 1u << k;
+                        if (z >= thr_hi) mmax |= 1u << k;
+                    }
+                    if (!(need & 1)) mmax = 0;
+                    uint32_t mall = mmin | mmax;
+                    while (mall) {
+                        const int k = __ffs(mall) - 1;
+                        mall &= mall - 1;
+                        const int tag = bk | (((mmin >> k) & 1) ? 4 : 0) | (((mmax >> k) & 1) ? 8 : 0);
+                        const int col = c * 32 + k;
+                        const int slot = atomicAdd(&M->qcount[qw], 1);
+                        if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
+                        if (slot < kQCap && nmine < 4) {
 #pragma unroll
-                        for (int k = 0; k < 32; k++) {
-                            const float z = __uint_as_float(v[k]);
-                            if (z <= thr_lo) mmin |= 1u << k;
-                            if ((need & 1) && z >= thr_hi) mmax |= 1u << k;
-                        }
-                        uint32_t mall = mmin | mmax;
-                        while (mall) {
-                            const int k = __ffs(mall) - 1;
-                            mall &= mall - 1;
-                            const bool cmin = (mmin >> k) & 1, cmax = (mmax >> k) & 1;
-                            const int col = c * 32 + k;
-                            const int slot = atomicAdd(&M->qcount[qw], 1);
-                            const int tag = bk | (cmin ? 4 : 0) | (cmax ? 8 : 0);
-                            if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
-                            if (slot < kQCap && nmine < 8) {
-                                myslot[nmine] = slot;
-                                mytag[nmine] = tag;
-                                nmine++;
-                            } else {
-                                // no room to track the job: recompute in place
-                                const float ze = exact_z(stg, row, col, Gf, g);
+                            for (int m = 0; m < 4; m++)
+                                if (m == nmine) {
+                                    ms[m] = slot;
+                                    mt[m] = tag;
+                                }
+                            nmine++;
+                        } else {
+                            const float ze = exact_z(stg, row, col, Gf, g);
 #pragma unroll
-                                for (int q = 0; q < 4; q++)
-                                    if (q == bk) {
-                                        if (cmin) ex_mn[q] = fminf(ex_mn[q], ze);
-                                        if (cmax) ex_mx[q] = fmaxf(ex_mx[q], ze);
-                                    }
-                            }
+                            for (int q = 0; q < 4; q++)
+                                if (q == bk) {
+                                    if (tag & 4) ex_mn[q] = fminf(ex_mn[q], ze);
+                                    if (tag & 8) ex_mx[q] = fmaxf(ex_mx[q], ze);
+                                }
                         }
                     }
                 }
@@ -532,15 +555,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     qjob[2 * j + 1] = __float_as_uint(exact_z(stg, (int)(jb & 0xffu), (int)(jb >> 8), Gf, g));
                 }
                 __syncwarp();
-                for (int m = 0; m < nmine; m++) {
-                    const float ze = __uint_as_float(qjob[2 * myslot[m] + 1]);
-                    const int tag = mytag[m];
 #pragma unroll
-                    for (int q = 0; q < 4; q++)
-                        if (q == (tag & 3)) {
-                            if (tag & 4) ex_mn[q] = fminf(ex_mn[q], ze);
-                            if (tag & 8) ex_mx[q] = fmaxf(ex_mx[q], ze);
-                        }
+                for (int m = 0; m < 4; m++) {
+                    if (m < nmine) {
+                        const float ze = __uint_as_float(qjob[2 * ms[m] + 1]);
+                        const int tag = mt[m];
+#pragma unroll
+                        for (int q = 0; q < 4; q++)
+                            if (q == (tag & 3)) {
+                                if (tag & 4) ex_mn[q] = fminf(ex_mn[q], ze);
+                                if (tag & 8) ex_mx[q] = fmaxf(ex_mx[q], ze);
+                            }
+                    }
                 }
                 __syncwarp();
 #pragma unroll
@@ -552,73 +578,121 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     }
                 }
             }
-#pragma unroll
-            for (int bk = 0; bk < 4; bk++)
-                if (bk < nbk && valid && (h_is_inf(s16[bk]) || h_is_inf(m16[bk]))) flag |= CG_FLAG_FP16_OVERFLOW;
 
-            // ---- 5. codes (fast path) with boundary check, packed into the row stage
+            // ---- 5. code parameters per block
+            float rinv[4], c0[4], lim[4];
+            int fast = 0;  // bit bk: no value of the block can leave [0, qmax]
+            int live = 0;  // bit bk: finite, non-zero scale (else every code is 0)
+#pragma unroll
+            for (int bk = 0; bk < 4; bk++) {
+                rinv[bk] = c0[bk] = 0.0f;
+                lim[bk] = 0.5f;
+                if (bk < nbk) {
+                    if (valid && (h_is_inf(s16[bk]) || h_is_inf(m16[bk]))) flag |= CG_FLAG_FP16_OVERFLOW;
+                    const float sc = h2f_bits(s16[bk]), mz = h2f_bits(m16[bk]);
+                    if (sc != 0.0f && !h_is_inf(s16[bk]) && !h_is_inf(m16[bk])) {
+                        const float r = __frcp_rn(sc);
+                        const float cc = -mz * r;
+                        rinv[bk] = r;
+                        c0[bk] = cc;
+                        // |t~ - t|: the value bound E/s, plus the rounding of rcp, c0 and the fma
+                        // (a few ulps of |z r| + |c0|) and of the definition's subtract and divide
+                        const float zr = fmaxf(fabsf(mn[bk]), fabsf(mx[bk])) * r;
+                        const float mu = E[bk] * r * 1.0001f + (zr + fabsf(cc) + qmaxf + 1.0f) * 4.8e-7f;
+                        lim[bk] = 0.5f - mu;
+                        const float tlo = (mn[bk] - E[bk]) * r + cc, thi = (mx[bk] + E[bk]) * r + cc;
+                        if (tlo > -0.49f + mu && thi < qmaxf + 0.49f - mu) fast |= 1 << bk;
+                        live |= 1 << bk;
+                    }
+                }
+            }
+
+            // ---- 6. codes from z~, stored straight from registers; near-boundary values queued
+            uint8_t* crow = a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
+            int nmine = 0;
+            int ms[4] = {0, 0, 0, 0}, mt[4] = {0, 0, 0, 0};
             if (lane == 0) M->qcount[qw] = 0;
             __syncwarp();
-            nmine = 0;
-#pragma unroll
             for (int c = 0; c < 4; c++) {
                 uint32_t v[32];
                 tmem_ld32(tacc + c * 32, v);
                 tmem_wait_ld();
                 const int bk = (c * 32) / blk;
-                float sc = 0.0f, mz = 0.0f, E = 0.0f;
-                uint32_t s16b = 0;
+                const float r = pick4(rinv, bk), cc = pick4(c0, bk), lm = pick4(lim, bk);
+                const bool fst = (fast >> bk) & 1;
+                const bool lv = (live >> bk) & 1;
+                uint32_t qv[32];
+                float dmax = 0.0f;
+                if (fst) {
 #pragma unroll
-                for (int q = 0; q < 4; q++)
-                    if (q == bk) {
-                        s16b = s16[q];
-                        mz = h2f_bits(m16[q]);
-                        E = Eb[q];
+                    for (int k = 0; k < 32; k++) {
+                        const float t = fmaf(__uint_as_float(v[k]), r, cc);
+                        const float y = t + kMagic;
+                        dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
+                        qv[k] = __float_as_uint(y);
                     }
-                sc = h2f_bits(s16b);
-                const bool zero_scale = (sc == 0.0f);
-                const float rinv = zero_scale ? 0.0f : __frcp_rn(sc);
-                const float mu = zero_scale ? 0.0f : E * rinv * 1.0001f + (qmaxf + 1.0f) * 4.8e-7f;
-                const float lim = 0.5f - mu;
+                } else {
+#pragma unroll
+                    for (int k = 0; k < 32; k++) {
+                        float t = fmaf(__uint_as_float(v[k]), r, cc);
+                        t = fminf(fmaxf(t, 0.0f), qmaxf);
+                        const float y = t + kMagic;
+                        dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
+                        qv[k] = lv ? __float_as_uint(y) : 0u;
+                    }
+                }
                 uint32_t words[BITS];
 #pragma unroll
                 for (int w = 0; w < BITS; w++) words[w] = 0;
-                uint32_t ambmask = 0;
 #pragma unroll
                 for (int k = 0; k < 32; k++) {
-                    const float z = __uint_as_float(v[k]);
-                    float t = __fmul_rn(__fsub_rn(z, mz), rinv);
-                    t = fminf(fmaxf(t, 0.0f), qmaxf);
-                    const float rt = rintf(t);
-                    const uint32_t q = zero_scale ? 0u : (uint32_t)(int)rt;
-                    if (fabsf(t - rt) > lim && !zero_scale) ambmask |= 1u << k;
+                    const uint32_t q = qv[k] & (uint32_t)qmax;
                     const int bit = k * BITS;
                     words[bit >> 5] |= q << (bit & 31);
                     if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
                 }
+                if (valid) {
+                    uint32_t* dst = reinterpret_cast<uint32_t*>(crow) + c * BITS;
+                    if (BITS % 4 == 0) {
 #pragma unroll
-                for (int w = 0; w < BITS; w++) my_codes[c * BITS + w] = words[w];
-                if (!valid) ambmask = 0;
-                while (ambmask) {
-                    const int k = __ffs(ambmask) - 1;
-                    ambmask &= ambmask - 1;
-                    const int col = c * 32 + k;
-                    const int slot = atomicAdd(&M->qcount[qw], 1);
-                    if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
-                    if (slot < kQCap && nmine < 8) {
-                        myslot[nmine] = slot;
-                        mytag[nmine] = col | ((int)s16b << 8);
-                        nmine++;
+                        for (int w = 0; w < BITS; w += 4)
+                            *reinterpret_cast<uint4*>(dst + w) = make_uint4(words[w], words[w + 1], words[w + 2], words[w + 3]);
+                    } else if (BITS % 2 == 0) {
+#pragma unroll
+                        for (int w = 0; w < BITS; w += 2) *reinterpret_cast<uint2*>(dst + w) = make_uint2(words[w], words[w + 1]);
                     } else {
-                        const float ze = exact_z(stg, row, col, Gf, g);
-                        const uint32_t q = quant_code(ze, sc, mz, qmax);
-                        const int bit = col * BITS;
-                        uint32_t* wp = my_codes + (bit >> 5);
-                        const uint32_t msk = (uint32_t)qmax;
-                        wp[0] = (wp[0] & ~(msk << (bit & 31))) | (q << (bit & 31));
-                        if ((bit & 31) + BITS > 32) {
-                            const int sh = 32 - (bit & 31);
-                            wp[1] = (wp[1] & ~(msk >> sh)) | (q >> sh);
+#pragma unroll
+                        for (int w = 0; w < BITS; w++) dst[w] = words[w];
+                    }
+                }
+                if (valid && lv && dmax > lm) {
+                    // rare: the values within the bound of a rounding boundary
+                    uint32_t amask = 0;
+#pragma unroll
+                    for (int k = 0; k < 32; k++) {
+                        float t = fmaf(__uint_as_float(v[k]), r, cc);
+                        if (!fst) t = fminf(fmaxf(t, 0.0f), qmaxf);
+                        const float y = t + kMagic;
+                        if (fabsf(t - (y - kMagic)) > lm) amask |= 1u << k;
+                    }
+                    while (amask) {
+                        const int k = __ffs(amask) - 1;
+                        amask &= amask - 1;
+                        const int col = c * 32 + k;
+                        const int slot = atomicAdd(&M->qcount[qw], 1);
+                        if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
+                        if (slot < kQCap && nmine < 4) {
+#pragma unroll
+                            for (int m = 0; m < 4; m++)
+                                if (m == nmine) {
+                                    ms[m] = slot;
+                                    mt[m] = col;
+                                }
+                            nmine++;
+                        } else {
+                            const float ze = exact_z(stg, row, col, Gf, g);
+                            const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
+                            patch_code<BITS>(crow, col * BITS, q);
                         }
                     }
                 }
@@ -631,45 +705,29 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     qjob[2 * j + 1] = __float_as_uint(exact_z(stg, (int)(jb & 0xffu), (int)(jb >> 8), Gf, g));
                 }
                 __syncwarp();
-                for (int m = 0; m < nmine; m++) {
-                    const float ze = __uint_as_float(qjob[2 * myslot[m] + 1]);
-                    const int col = mytag[m] & 0xff;
-                    const uint32_t s16b = (uint32_t)mytag[m] >> 8;
-                    const int bk = col / blk;
-                    float mz = 0.0f;
 #pragma unroll
-                    for (int q = 0; q < 4; q++)
-                        if (q == bk) mz = h2f_bits(m16[q]);
-                    const uint32_t q = quant_code(ze, h2f_bits(s16b), mz, qmax);
-                    const int bit = col * BITS;
-                    uint32_t* wp = my_codes + (bit >> 5);
-                    const uint32_t msk = (uint32_t)qmax;
-                    wp[0] = (wp[0] & ~(msk << (bit & 31))) | (q << (bit & 31));
-                    if ((bit & 31) + BITS > 32) {
-                        const int sh = 32 - (bit & 31);
-                        wp[1] = (wp[1] & ~(msk >> sh)) | (q >> sh);
+                for (int m = 0; m < 4; m++) {
+                    if (m < nmine) {
+                        const float ze = __uint_as_float(qjob[2 * ms[m] + 1]);
+                        const int col = mt[m];
+                        const int bk = col / blk;
+                        const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
+                        patch_code<BITS>(crow, col * BITS, q);
                     }
                 }
             }
-            __syncwarp();
 
-            // ---- 6. stores
+            // ---- 7. scales; release the stage and the accumulator buffer
             if (valid) {
-                const int64_t t = t0 + row;
-                uint4* dstc = reinterpret_cast<uint4*>(a.codes + a.cmap.at(l, s, b, h, t));
-#pragma unroll
-                for (int w = 0; w < kWords / 4; w++)
-                    dstc[w] = make_uint4(my_codes[4 * w], my_codes[4 * w + 1], my_codes[4 * w + 2], my_codes[4 * w + 3]);
-                uint32_t* dsts = a.scales + a.smap.at(l, s, b, h, t);
+                uint32_t* sp = a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
 #pragma unroll
                 for (int bk = 0; bk < 4; bk++)
-                    if (bk < nbk) dsts[bk] = s16[bk] | (m16[bk] << 16);
+                    if (bk < nbk) sp[bk] = s16[bk] | (m16[bk] << 16);
             }
-            // ---- 7. release the accumulator buffer and the stage
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
-                mbar_arrive(&M->acc_empty[buf]);
+                mbar_arrive(&M->accempty[buf]);
                 mbar_arrive(&M->empty[st]);
             }
         }
@@ -684,25 +742,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     }
 }
 
-int num_sms() {
-    static int n[64] = {};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 0 || dev >= 64) return 148;
-    if (!n[dev]) {
-        int v = 0;
-        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
-        n[dev] = v > 0 ? v : 148;
-    }
-    return n[dev];
-}
-
 template <int BITS>
 cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
     const size_t smem = EncSmem::total + 1024;
     cudaError_t e = cudaFuncSetAttribute(tc_encode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const int64_t grid = P.n_tiles < num_sms() ? P.n_tiles : num_sms();
+    const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
     tc_encode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(map, P);
     return cudaGetLastError();
 }
@@ -715,18 +760,16 @@ bool tc_row_encode_eligible(const RowArgs& a) {
     if (a.t_count < 64) return false;
     const int64_t rows = (int64_t)a.L * 2 * a.B * a.H * a.T_x;
     if (rows + 128 >= (int64_t)1 << 31) return false;
-    if (reinterpret_cast<uintptr_t>(a.x) & 15u) return false;
+    if ((reinterpret_cast<uintptr_t>(a.x) & 15u) || (reinterpret_cast<uintptr_t>(a.codes) & 15u)) return false;
     return tmap_encode_fn() != nullptr;
 }
 
 cudaError_t tc_launch_row_encode(const RowArgs& a, cudaStream_t st) {
     EncParams P;
     P.a = a;
+    P.S = tc::make_sched(a);
     P.npass = a.g == 128 ? 2 : 3;
-    P.n_units = (int64_t)a.L * a.s_n * a.B * a.H;
-    P.tiles_per_unit = (a.t_count + 127) / 128;
-    P.n_tiles = P.n_units * P.tiles_per_unit;
-    if (P.n_tiles == 0) return cudaSuccess;
+    if (P.S.n_tiles == 0) return cudaSuccess;
     CUtensorMap map;
     const uint64_t rows = (uint64_t)a.L * 2 * a.B * a.H * a.T_x;
     if (!make_tmap_bf16_sw128(&map, a.x, rows, kD, kD * 2, 128)) return cudaErrorInvalidValue;

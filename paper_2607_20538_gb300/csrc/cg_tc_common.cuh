@@ -51,6 +51,60 @@ __device__ __forceinline__ TileInfo tile_info(const RowArgs& a, const Sched& S, 
     return ti;
 }
 
+// Walks a CTA's tile range in steps of 1 or 2 tiles without integer division (the full
+// decomposition is done once, at init).
+struct TileIter {
+    int tt;        // tile within the unit
+    int tpu;       // tiles per unit
+    int l, s, b, h;
+    int64_t seg;
+
+    __device__ __forceinline__ void init(const RowArgs& a, const Sched& S, int64_t tile) {
+        const TileInfo ti = tile_info(a, S, tile);
+        tpu = (int)S.tiles_per_unit;
+        tt = (int)(ti.t0 >> 7);
+        l = ti.l;
+        s = ti.s;
+        b = ti.b;
+        h = ti.h;
+        seg = ti.seg;
+    }
+    __device__ __forceinline__ void next_unit(const RowArgs& a) {
+        if (++b == a.B) {
+            b = 0;
+            seg++;
+            if (++h == a.H) {
+                h = 0;
+                if (++s == a.s_lo + a.s_n) {
+                    s = a.s_lo;
+                    l++;
+                }
+            }
+        }
+    }
+    __device__ __forceinline__ void step(const RowArgs& a, int k) {
+        tt += k;
+        while (tt >= tpu) {
+            tt -= tpu;
+            next_unit(a);
+        }
+    }
+    // last tile of its gauge segment (the segment's units are B consecutive units)
+    __device__ __forceinline__ bool seg_last(const RowArgs& a) const { return tt == tpu - 1 && b == a.B - 1; }
+    __device__ __forceinline__ TileInfo info(const RowArgs& a) const {
+        TileInfo ti;
+        ti.l = l;
+        ti.s = s;
+        ti.b = b;
+        ti.h = h;
+        ti.seg = seg;
+        ti.t0 = (int64_t)tt * 128;
+        const int64_t left = a.t_count - ti.t0;
+        ti.rows_valid = (int)(left < 128 ? left : 128);
+        return ti;
+    }
+};
+
 // Row of unit (l, s, b, h) in the dense [L][2][B][H][T_x][d] tensor.
 __device__ __forceinline__ int64_t dense_row(const RowArgs& a, const TileInfo& ti) {
     return (((int64_t)(ti.l * 2 + ti.s) * a.B + ti.b) * a.H + ti.h) * a.T_x + ti.t0;

@@ -146,13 +146,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
         // ------------------------------------------------------------ codes producer
         if (lane == 0 && my_tiles > 0) {
             int issued = 0;
-            for (int i = 0; i < my_tiles; i++) {
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
                 const int st = i % kCStages;
                 if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
                     *abort_flag = 1;
                     break;
                 }
-                const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+                const tc::TileInfo ti = it.info(a);
                 const uint32_t bytes = (uint32_t)ti.rows_valid * kRowBytes;
                 mbar_arrive_expect_tx(&M->cfull[st], bytes);
                 bulk_load(cst + st * kCStageBytes, a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0), bytes,
@@ -172,8 +174,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             const uint32_t idesc = idesc_bf16_f32(128, gb);
             int64_t cur = -1;
             int committed = 0;
-            for (int i = 0; i < my_tiles; i++) {
-                const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+                const tc::TileInfo ti = it.info(a);
                 const int64_t ls = ti.seg - seg0;
                 bool ok = true;
                 if (ti.seg != cur) {
@@ -209,8 +213,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                 }
                 mma_commit(&M->accfull[buf]);
                 mma_commit(&M->aempty[ab]);
-                const bool last_of_seg =
-                    (i + 1 == my_tiles) || tc::tile_info(a, S, t_begin + i + 1).seg != ti.seg;
+                const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
                 if (last_of_seg) mma_commit(&M->bfree);
                 committed = i + 1;
             }
@@ -226,8 +229,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
         const int row = uw * 32 + lane;
         int64_t cur = -1;
         int nconv = 0;
-        for (int i = 0; i < my_tiles; i++) {
-            const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+        tc::TileIter it;
+        it.init(a, S, t_begin);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            const tc::TileInfo ti = it.info(a);
             if (ti.seg != cur) {
                 const int64_t ls = ti.seg - seg0;
                 if (nconv > 0) {
@@ -308,8 +313,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
         // ------------------------------------------------------------ epilogue
         const int ew = warp & 3;
         const int row = ew * 32 + lane;
-        for (int i = 0; i < my_tiles; i++) {
-            const tc::TileInfo ti = tc::tile_info(a, S, t_begin + i);
+        tc::TileIter it;
+        it.init(a, S, t_begin);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
             const int buf = i & 1;
             bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
