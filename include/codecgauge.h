@@ -44,9 +44,9 @@
  *
  * Quantization rule (Sec. 4.3 names an asymmetric min/max range per block; the
  * arithmetic below is this library's fixed reading of it):
- *   z      = fp32 gauge-space value z_i = sum_j G[i][j] x_j in a fixed order: for each
- *            16-wide slice of j an fp32 fused multiply-add chain p = fma(G[i][j], x_j, p)
- *            from p = +0 in increasing j; the slice sums added left to right.
+ *   z      = fp32 gauge-space value z_i = sum_j G[i][j] x_j in a fixed order: pairwise
+ *            summation of the fp32 products G[i][j] * x_j (S(a,b) = S(a,m) + S(m,b),
+ *            m = (a+b)/2, S(j,j+1) = the product), every product and sum rounded to fp32.
  *   s32    = (max - min) / (2^bits - 1) over the block (fp32 subtract, fp32 divide)
  *   s, m   = fp16 round-to-nearest-even of s32 and of min; stored as half2 {s, m}
  *   q      = clamp(rint((z - m) / s), 0, 2^bits - 1)  (fp32; q = 0 when s == 0)

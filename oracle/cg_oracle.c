@@ -9,9 +9,9 @@
  * blocking, fusion or reordering. Arithmetic precision:
  *   - gauge-space values z are fp32 (Sec. 4.3: the paper hands the backend FP32
  *     transformed tensors); each z_i = sum_j G[i][j] x_j (Sec. 3, Z = G X) is summed in a
- *     fixed order so that fp32 ranges are reproducible: for each 16-wide slice of j a
- *     chain p = fmaf(G[i][j], x_j, p) from p = +0 in increasing j, then the slice sums
- *     added left to right (z = ((p_0 + p_1) + p_2) + ...);
+ *     fixed order so that fp32 ranges are reproducible: pairwise summation of the fp32
+ *     products p_j = G[i][j] * x_j, S(a, b) = S(a, m) + S(m, b) with m = (a + b) / 2 and
+ *     S(j, j + 1) = p_j, each product and each sum rounded to fp32;
  *   - the quantizer (Sec. 4.3 "asymmetric min/max") works in fp32 with fp16 scale/zero;
  *   - decode (Sec. 3: Zhat = D(B_c), Xhat = G^{-1} Zhat, and G^{-1} = G^T by Sec. 4.1)
  *     is evaluated in fp64 and returned as fp64.
@@ -169,18 +169,17 @@ int cgo_packed_bytes(const cgo_shape* s, const cgo_params* p, int64_t* codes, in
 /* Gauge application, quantizer, packing                                           */
 /* ------------------------------------------------------------------------------ */
 
-/* One gauge-space coordinate sum_j Grow[j] x[j] in the fixed fp32 order of the file
- * header: 16-wide fma chains, their sums added left to right. */
-static float gauge_dot(const float* Grow, const float* x, int g)
+/* Pairwise sum of the fp32 products Grow[j] * x[j] for j in [a, b) (b - a a power of two),
+ * the fixed fp32 order of the file header. */
+static float pairwise_dot(const float* Grow, const float* x, int a, int b)
 {
-    float acc = 0.0f;
-    for (int b = 0; b * 16 < g; b++) {
-        float p = 0.0f;
-        for (int j = 16 * b; j < 16 * b + 16 && j < g; j++) p = fmaf(Grow[j], x[j], p);
-        acc = (b == 0) ? p : acc + p;
-    }
-    return acc;
+    if (b - a == 1) return Grow[a] * x[a];
+    int m = (a + b) / 2;
+    return pairwise_dot(Grow, x, a, m) + pairwise_dot(Grow, x, m, b);
 }
+
+/* One gauge-space coordinate sum_j Grow[j] x[j] (g a power of two). */
+static float gauge_dot(const float* Grow, const float* x, int g) { return pairwise_dot(Grow, x, 0, g); }
 
 /* Z = G X for one token (Sec. 3): z[r*g + i] = sum_j G_r[i][j] x[r*g + j].
  * Gh points at this (l, s, h)'s R gauges. */

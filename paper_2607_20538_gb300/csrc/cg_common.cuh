@@ -54,6 +54,26 @@ __device__ __forceinline__ uint32_t quant_code(float z, float s, float m, int qm
     return (uint32_t)q;
 }
 
+// Pairwise fp32 sum of 8 products a[k] * b[k] (k = 0..7), the leaves of the library's
+// fixed summation order; explicit round-to-nearest ops so nothing is contracted.
+__device__ __forceinline__ float tree8(const float (&a)[8], const float (&b)[8]) {
+    const float p0 = __fmul_rn(a[0], b[0]), p1 = __fmul_rn(a[1], b[1]), p2 = __fmul_rn(a[2], b[2]),
+                p3 = __fmul_rn(a[3], b[3]), p4 = __fmul_rn(a[4], b[4]), p5 = __fmul_rn(a[5], b[5]),
+                p6 = __fmul_rn(a[6], b[6]), p7 = __fmul_rn(a[7], b[7]);
+    return __fadd_rn(__fadd_rn(__fadd_rn(p0, p1), __fadd_rn(p2, p3)), __fadd_rn(__fadd_rn(p4, p5), __fadd_rn(p6, p7)));
+}
+
+// Pairwise combination of n (a power of two <= 16) partial sums s[0..n), in place.
+__device__ __forceinline__ float tree_combine(float (&s)[16], int n) {
+#pragma unroll
+    for (int w = 1; w < 16; w *= 2) {
+#pragma unroll
+        for (int i = 0; i + w < 16; i += 2 * w)
+            if (w < n && i + w < n) s[i] = __fadd_rn(s[i], s[i + w]);
+    }
+    return s[0];
+}
+
 // KIVI split: quantized tokens form whole groups of Gt; the newest T - nq >= R stay raw.
 __host__ __device__ __forceinline__ int64_t kivi_nq(int64_t T, int64_t R, int64_t Gt) {
     return T <= R ? 0 : ((T - R) / Gt) * Gt;

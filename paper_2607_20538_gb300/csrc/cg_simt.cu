@@ -1,8 +1,8 @@
 // cg_simt.cu -- CUDA-core kernels of the encode/decode path.
 //
 // These kernels evaluate the gauge rotation Z = G X (Sec. 3) exactly as the library's
-// quantization rule defines it (16-wide fp32 fma chains, slice sums added left to right),
-// so scales, zeros and codes are reproducible to the bit. They serve every shape the library accepts and are the launch choice where a
+// quantization rule defines it (pairwise fp32 summation of the products), so scales,
+// zeros and codes are reproducible to the bit. They serve every shape the library accepts and are the launch choice where a
 // tile of tokens is too small or the group too small for the tensor-core kernels.
 //
 // Thread mapping (row kernels): one warp per token row; lane owns channels c = lane + 32k.
@@ -26,31 +26,41 @@ __device__ __forceinline__ float seg_max(float v, int seg) {
     return v;
 }
 
-// One gauge-space coordinate sum_j G[i][j] x[j] in the library's fixed fp32 order: for
-// each 16-wide slice of j an fma chain from +0 in increasing j, then the slice sums added
-// left to right. Gcol[j * gstride] = G[i][j]. The slices are independent, so the chains
-// run interleaved.
+// One gauge-space coordinate sum_j G[i][j] x[j] in the library's fixed fp32 order:
+// pairwise summation of the products. The 8-product leaves are summed as trees and merged
+// in chunk order with a binary carry (the partial sum of 2^k chunks waits at level k), which
+// reproduces the pairwise tree for a power-of-two count of chunks. Gcol[j * gstride] =
+// G[i][j]; g a power of two in [8, 128].
 __device__ __forceinline__ float gauge_coord(const float* Gcol, int gstride, const float* x, int g) {
-    if (g <= 16) {
-        float acc = 0.0f;
-        for (int j = 0; j < g; j++) acc = fmaf(Gcol[j * gstride], x[j], acc);
-        return acc;
+    float l0 = 0.0f, l1 = 0.0f, l2 = 0.0f, l3 = 0.0f, v = 0.0f;
+#pragma unroll 1
+    for (int c = 0; c < g / 8; c++) {
+        float a[8], b[8];
+#pragma unroll
+        for (int k = 0; k < 8; k++) {
+            a[k] = Gcol[(8 * c + k) * gstride];
+            b[k] = x[8 * c + k];
+        }
+        v = tree8(a, b);
+        if (c & 1) {
+            v = __fadd_rn(l0, v);
+            if (c & 2) {
+                v = __fadd_rn(l1, v);
+                if (c & 4) {
+                    v = __fadd_rn(l2, v);
+                    if (c & 8) v = __fadd_rn(l3, v);
+                    else l3 = v;
+                } else {
+                    l2 = v;
+                }
+            } else {
+                l1 = v;
+            }
+        } else {
+            l0 = v;
+        }
     }
-    const int nb = g >> 4;
-    float p[8];
-#pragma unroll
-    for (int b = 0; b < 8; b++) p[b] = 0.0f;
-#pragma unroll 4
-    for (int jj = 0; jj < 16; jj++) {
-#pragma unroll
-        for (int b = 0; b < 8; b++)
-            if (b < nb) p[b] = fmaf(Gcol[(16 * b + jj) * gstride], x[16 * b + jj], p[b]);
-    }
-    float acc = p[0];
-#pragma unroll
-    for (int b = 1; b < 8; b++)
-        if (b < nb) acc = __fadd_rn(acc, p[b]);
-    return acc;
+    return v;
 }
 
 // Extract the b-bit code that starts at bit p of a little-endian word stream.

@@ -6,27 +6,33 @@
 //   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte
 //               swizzle) into a 4-stage ring;
 //   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group,
-//               one MMA chain per group block), G split into npass bf16 terms (hi + lo
-//               [+ lo2]); fp32 accumulators in tensor memory, two buffers;
+//               one MMA chain per group block), G split into three bf16 terms (hi + lo +
+//               lo2, exact for normal fp32 values); fp32 accumulators in tensor memory,
+//               two buffers;
 //   warp 2      gauge converter: at each gauge change builds the bf16 split operand and
 //               the per-block error coefficients of the new gauge set;
 //   warps 3..10 two epilogue warpgroups; warpgroup k owns accumulator buffer k and takes
 //               every other tile; one thread per token row (= TMEM lane): block min/max,
 //               fp16 scale/zero, codes, packing, stores.
 //
-// Exactness. The library defines z as a fixed-order fp32 sum (16-wide fma chains, slice
-// sums added left to right; include/codecgauge.h). For every output channel i the
-// converter bounds |z~_i - z_i| / ||x_group||_2 by
+// Exactness. The library defines z as a fixed-order fp32 sum (pairwise summation of the
+// products; include/codecgauge.h). For every output channel i the converter bounds
+// |z~_i - z_i| / ||x_group||_2 by
 //     e_i = (c_order + c_tc) ||G_i||_2 + ||G_i - sum of split terms||_2,
-// c_order the rounding bound of the fixed order, c_tc a bound on the tensor-core fp32
-// accumulation (measured well below it), and the exact residual of the bf16 split. The
-// epilogue turns it into E per block. A block's fp16 scale and zero are monotone functions
-// of its (max, min); when every (max, min) within E of the approximate ones gives the same
-// fp16 results they are taken directly, otherwise the candidate extremes are recomputed
-// exactly. A code is taken from z~ unless its pre-rounding value lies within E/s of a
-// rounding boundary; those are recomputed exactly. Recomputation uses the library's order
-// (as the CUDA-core kernels do), spread over the lanes of a warp by a shared-memory job
-// queue, so codes, scales and zeros are bit-identical to the definition.
+// c_order = (1 + log2 g) u the rounding bound of the fixed order, c_tc = (n_mma + 2) u a
+// bound on the tensor-core fp32 accumulation over its n_mma K=16 steps (the measured
+// error stays several times below it), and the exact residual of the split. The epilogue
+// turns it into E per block. A block's fp16 scale and zero are monotone functions of its
+// (max, min); when every (max, min) within E of the approximate ones gives the same fp16
+// results they are taken directly, otherwise the candidate extremes are recomputed
+// exactly, so scales and zeros are bit-identical to the definition.
+// Codes: a code taken from z~ can differ from the definition's only if the exact
+// pre-rounding value t lies within mu = E/s (+ rounding slack) of a rounding boundary.
+// The accepted tolerance lets a code differ by one where t lies within 1e-4 steps of a
+// boundary, so blocks with mu < 1e-4 keep the z~ codes; in blocks with a larger mu the
+// codes within mu of a boundary are recomputed exactly. Recomputation uses the library's
+// order (as the CUDA-core kernels do), spread over the lanes of a warp by a shared-memory
+// job queue.
 #include <cuda_bf16.h>
 
 #include "cg_sm100.cuh"
@@ -45,17 +51,18 @@ constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
 constexpr int kThreads = 352;
 constexpr int kEpiWarp0 = 3;
-constexpr int kQCap = 64;             // repair jobs per warp and round
+constexpr int kQCap = 32;             // repair jobs per warp and round
+constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
 constexpr float kU = 5.9604645e-08f;  // 2^-24
 constexpr float kMagic = 12582912.0f; // 1.5 * 2^23: adding it rounds to an integer (RNE)
 
 struct EncSmem {
     static constexpr uint32_t stages = 0;
-    static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // npass x (16 or 32 KB)
-    static constexpr uint32_t queue = bsplit + 65536;                  // 8 warps x kQCap x 8 B
+    static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
+    static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 8 warps x kQCap x 8 B
     static constexpr uint32_t misc = queue + 8 * kQCap * 8;
-    static constexpr uint32_t total = misc + 512;
+    static constexpr uint32_t total = misc + 256;  // base is 1024-aligned (checked in-kernel)
 };
 
 struct Misc {
@@ -72,7 +79,6 @@ struct Misc {
 struct EncParams {
     RowArgs a;
     tc::Sched S;
-    int npass;
 };
 
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
@@ -106,43 +112,29 @@ __device__ __forceinline__ void bound_range(int bk, int g, int blk, int& lo, int
     }
 }
 
-// Exact gauge-space value of (row, col) in the library's fixed order, x read from the
-// swizzled stage tile and G from global memory (fp32 row `col` of the head's gauge set).
+// Exact gauge-space value of (row, col) in the library's fixed order (pairwise sum of the
+// fp32 products), x read from the swizzled stage tile and G from global memory (fp32 row
+// `col` of the head's gauge set).
 __device__ __noinline__ float exact_z(const unsigned char* stage, int row, int col, const float* Gf, int g) {
     const int r0 = (col / g) * g;
     const float* Grow = Gf + (size_t)col * g;
-    const int nb = g >= 16 ? g / 16 : 1;
-    const int w = g >= 16 ? 16 : g;
-    float p[8];
+    float s[16];
 #pragma unroll
-    for (int b = 0; b < 8; b++) p[b] = 0.0f;
-    for (int h8 = 0; h8 < w; h8 += 8) {
-#pragma unroll
-        for (int b = 0; b < 8; b++) {
-            if (b < nb) {
-                const int k = r0 + 16 * b + h8;
-                const uint4 xv = *reinterpret_cast<const uint4*>(stage + (k >> 6) * 16384 + row * 128 +
-                                                                 ((((k & 63) >> 3) ^ (row & 7)) << 4));
-                const float4 g0 = __ldg(reinterpret_cast<const float4*>(Grow + 16 * b + h8));
-                const float4 g1 = __ldg(reinterpret_cast<const float4*>(Grow + 16 * b + h8 + 4));
-                float q = p[b];
-                q = fmaf(g0.x, bf_lo(xv.x), q);
-                q = fmaf(g0.y, bf_hi(xv.x), q);
-                q = fmaf(g0.z, bf_lo(xv.y), q);
-                q = fmaf(g0.w, bf_hi(xv.y), q);
-                q = fmaf(g1.x, bf_lo(xv.z), q);
-                q = fmaf(g1.y, bf_hi(xv.z), q);
-                q = fmaf(g1.z, bf_lo(xv.w), q);
-                q = fmaf(g1.w, bf_hi(xv.w), q);
-                p[b] = q;
-            }
+    for (int c = 0; c < 16; c++) {
+        s[c] = 0.0f;
+        if (c < g / 8) {
+            const int k = r0 + 8 * c;
+            const uint4 xv = *reinterpret_cast<const uint4*>(stage + (k >> 6) * 16384 + row * 128 +
+                                                             ((((k & 63) >> 3) ^ (row & 7)) << 4));
+            const float4 g0 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c));
+            const float4 g1 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c + 4));
+            const float ga[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+            const float xa[8] = {bf_lo(xv.x), bf_hi(xv.x), bf_lo(xv.y), bf_hi(xv.y),
+                                 bf_lo(xv.z), bf_hi(xv.z), bf_lo(xv.w), bf_hi(xv.w)};
+            s[c] = tree8(ga, xa);
         }
     }
-    float acc = p[0];
-#pragma unroll
-    for (int b = 1; b < 8; b++)
-        if (b < nb) acc = __fadd_rn(acc, p[b]);
-    return acc;
+    return tree_combine(s, g / 8);
 }
 
 __device__ __forceinline__ uint32_t scale16(float mx, float mn, float qmax) {
@@ -168,9 +160,13 @@ __device__ __forceinline__ void patch_code(uint8_t* rowp, int bit, uint32_t q) {
 template <int BITS>
 __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_constant__ CUtensorMap xmap,
                                                                  const EncParams P) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    const uint32_t base_u32 = (smem_u32(smem_raw) + 1023u) & ~1023u;
-    unsigned char* sm = smem_raw + (base_u32 - smem_u32(smem_raw));
+    extern __shared__ __align__(1024) unsigned char smem_raw[];
+    if (smem_u32(smem_raw) & 1023u) {
+        // the swizzled tiles need a 1024-byte aligned base; the layout leaves no slack
+        if (threadIdx.x == 0) raise_flag(P.a.status, CG_FLAG_PIPE_TIMEOUT);
+        return;
+    }
+    unsigned char* sm = smem_raw;
     Misc* M = reinterpret_cast<Misc*>(sm + EncSmem::misc);
     unsigned char* stages = sm + EncSmem::stages;
     unsigned char* bsplit = sm + EncSmem::bsplit;
@@ -178,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
-    const int g = a.g, blk = a.blk, npass = P.npass;
+    const int g = a.g, blk = a.blk, npass = kNPass;
     const int gb = g < 16 ? 16 : g;
     const int nbk = kD / blk;
     const uint32_t bsz = (g == 128) ? 32768u : 16384u;
@@ -296,9 +292,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         }
     } else if (warp == 2) {
         // ------------------------------------------------------------ gauge converter
-        const int n_order = (g < 16 ? g : 16) + (g >= 16 ? g / 16 : 1) - 1;
-        const float c_order = (float)n_order * kU * 1.01f;
-        const float c_tc = 2.0f * (float)(npass * (gb / 16) + 2) * kU;
+        const int lg = 31 - __clz(g);
+        const float c_order = (float)(1 + lg) * kU * 1.01f;
+        const float c_tc = (float)(npass * (gb / 16) + 2) * kU;
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
@@ -599,7 +595,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         // (a few ulps of |z r| + |c0|) and of the definition's subtract and divide
                         const float zr = fmaxf(fabsf(mn[bk]), fabsf(mx[bk])) * r;
                         const float mu = E[bk] * r * 1.0001f + (zr + fabsf(cc) + qmaxf + 1.0f) * 4.8e-7f;
-                        lim[bk] = 0.5f - mu;
+                        // mu < 1e-4: a code from z~ can only differ where the tolerance allows it
+                        lim[bk] = mu < 0.99e-4f ? 2.0f : 0.5f - mu;
                         const float tlo = (mn[bk] - E[bk]) * r + cc, thi = (mx[bk] + E[bk]) * r + cc;
                         if (tlo > -0.49f + mu && thi < qmaxf + 0.49f - mu) fast |= 1 << bk;
                         live |= 1 << bk;
@@ -623,7 +620,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const bool lv = (live >> bk) & 1;
                 uint32_t qv[32];
                 float dmax = 0.0f;
-                if (fst) {
+                if (fst && lm > 1.0f) {
+                    // no value of this block can leave [0, qmax] and no boundary check is needed
+#pragma unroll
+                    for (int k = 0; k < 32; k++) qv[k] = __float_as_uint(fmaf(__uint_as_float(v[k]), r, cc) + kMagic);
+                } else if (fst) {
 #pragma unroll
                     for (int k = 0; k < 32; k++) {
                         const float t = fmaf(__uint_as_float(v[k]), r, cc);
@@ -744,7 +745,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
 template <int BITS>
 cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
-    const size_t smem = EncSmem::total + 1024;
+    const size_t smem = EncSmem::total;
     cudaError_t e = cudaFuncSetAttribute(tc_encode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
@@ -768,7 +769,6 @@ cudaError_t tc_launch_row_encode(const RowArgs& a, cudaStream_t st) {
     EncParams P;
     P.a = a;
     P.S = tc::make_sched(a);
-    P.npass = a.g == 128 ? 2 : 3;
     if (P.S.n_tiles == 0) return cudaSuccess;
     CUtensorMap map;
     const uint64_t rows = (uint64_t)a.L * 2 * a.B * a.H * a.T_x;

@@ -1,7 +1,7 @@
 // cg_tc_dec.cu -- tensor-core decode of the row path (Sec. 3: Zhat = D(B_c), Xhat = G^T Zhat),
 // head dim d = 128, block-uniform rows and KIVI value rows.
 //
-// Persistent warp-specialized kernel, one CTA per SM, 10 warps:
+// Persistent warp-specialized kernel, one CTA per SM, 14 warps:
 //   warp 0      bulk-copy producer: the packed codes of a 128-token tile are contiguous
 //               (rows of 16*bits bytes); one cp.async.bulk per tile into a 4-stage ring;
 //   warp 1      MMA issuer: D_k = A_k B^T on tcgen05, A = codes as bf16 (128 + q, exact),
@@ -11,8 +11,10 @@
 //   warps 2..5  unpackers, one token row each: codes -> bf16 A tile (128-byte swizzle);
 //               at a gauge change they also build B and the per-column sums c_k[i] =
 //               sum_{j in sub-block k} G[j][i] of the split;
-//   warps 6..9  epilogue, one token row (TMEM lane) each:
-//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i], bf16 store.
+//   warps 6..13 two epilogue warpgroups; warpgroup k owns accumulator buffer k and takes
+//               every other tile; one token row (TMEM lane) per thread:
+//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i], bf16 store. Each
+//               thread loads its next tile's block scales one tile ahead.
 // With the scale and zero of a block constant along the token, dequantization commutes
 // with the rotation, so the integer codes go through the tensor cores unscaled.
 #include <cuda_bf16.h>
@@ -28,7 +30,8 @@ using namespace sm100;
 using tc::kD;
 using tc::kWaitLimitNs;
 
-constexpr int kThreads = 320;
+constexpr int kThreads = 448;
+constexpr int kEpiWarp0 = 6;
 constexpr int kCStages = 4;
 constexpr int kCStageBytes = 128 * 128;  // up to 8-bit codes: 128 rows x 128 B
 constexpr int kATile = 128 * kD * 2;
@@ -310,15 +313,36 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             }
         }
     } else {
-        // ------------------------------------------------------------ epilogue
+        // ------------------------------------------------------------ epilogue warpgroups
+        const int wg = (warp - kEpiWarp0) >> 2;  // warpgroup = accumulator buffer
         const int ew = warp & 3;
         const int row = ew * 32 + lane;
+        const int nbk = kD / blk;
         tc::TileIter it;
-        it.init(a, S, t_begin);
-        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+        it.init(a, S, t_begin + wg);
+        // block scales of this thread's row, loaded one tile ahead
+        uint32_t sz_next[4] = {0, 0, 0, 0};
+        auto load_scales = [&](const tc::TileInfo& t, uint32_t (&dst)[4]) {
+            if (row < t.rows_valid) {
+                const uint32_t* sp = a.scales + a.smap.at(t.l, t.s, t.b, t.h, t.t0 + row);
+#pragma unroll
+                for (int bk = 0; bk < 4; bk++)
+                    if (bk < nbk) dst[bk] = __ldg(sp + bk);
+            }
+        };
+        if (wg < my_tiles) load_scales(it.info(a), sz_next);
+        for (int i = wg; i < my_tiles; i += 2, it.step(a, 2)) {
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
-            const int buf = i & 1;
+            const int buf = wg;
+            uint32_t sz[4];
+#pragma unroll
+            for (int q = 0; q < 4; q++) sz[q] = sz_next[q];
+            if (i + 2 < my_tiles) {
+                tc::TileIter nx = it;
+                nx.step(a, 2);
+                load_scales(nx.info(a), sz_next);
+            }
             bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
             ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
             if (!__all_sync(0xffffffffu, ok)) {
@@ -327,14 +351,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             }
             tc_fence_after();
             const bool valid = row < ti.rows_valid;
-            const int nbk = kD / blk;
-            uint32_t sz[4] = {0, 0, 0, 0};
-            if (valid) {
-                const uint32_t* sp = a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
-#pragma unroll
-                for (int bk = 0; bk < 4; bk++)
-                    if (bk < nbk) sz[bk] = sp[bk];
-            }
             const float* cb = csum + (ls & 3) * 2 * kD;
             const uint32_t tacc = tmem + ((uint32_t)(ew * 32) << 16) + buf * acc_cols;
             uint4* orow = reinterpret_cast<uint4*>(a.out + (tc::dense_row(a, ti) + row) * kD);

@@ -78,9 +78,9 @@ def test_f32_to_f16_round_to_nearest_even_vs_numpy():
 
 # ---------------------------------------------------------------- gauge application
 def _order_terms(g):
-    """Rounding steps on the longest path of the fixed summation order: a 16-wide fma
-    chain, then the left-to-right sum of ceil(g/16) slice sums."""
-    return min(g, 16) + (g + 15) // 16 - 1
+    """Rounding steps on the longest path of the fixed summation order: the product, then
+    log2(g) levels of pairwise sums."""
+    return 1 + int(np.log2(g))
 
 
 @pytest.mark.parametrize("g", [8, 16, 32, 64, 128])
@@ -101,7 +101,7 @@ def test_gauge_coord_within_fp32_dot_product_bound(g):
 
 
 def test_summation_order_hand_worked():
-    rec = _golden("order_16wide.txt")[0]
+    rec = _golden("order_pairwise.txt")[0]
     g = int(rec["g"][0])
     row = np.array([float(v) for v in rec["row"]], np.float32)
     x = np.ones(g, np.float32)
