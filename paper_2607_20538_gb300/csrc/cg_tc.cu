@@ -8,12 +8,12 @@
 //   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group,
 //               one MMA chain per group block), G split into three bf16 terms (hi + lo +
 //               lo2, exact for normal fp32 values); fp32 accumulators in tensor memory,
-//               two buffers;
+//               four buffers (the MMA runs up to two tiles ahead of each warpgroup);
 //   warp 2      gauge converter: at each gauge change builds the bf16 split operand and
 //               the per-block error coefficients of the new gauge set;
-//   warps 3..10 two epilogue warpgroups; warpgroup k owns accumulator buffer k and takes
-//               every other tile; one thread per token row (= TMEM lane): block min/max,
-//               fp16 scale/zero, codes, packing, stores.
+//   warps 3..10 two epilogue warpgroups; warpgroup k takes every other tile; one thread
+//               per token row (= TMEM lane): block min/max, fp16 scale/zero, codes,
+//               packing, stores.
 //
 // Exactness. The library defines z as a fixed-order fp32 sum (pairwise summation of the
 // products; include/codecgauge.h). For every output channel i the converter bounds
@@ -52,6 +52,8 @@ constexpr int kTileBytes = 128 * kD * 2;
 constexpr int kThreads = 352;
 constexpr int kEpiWarp0 = 3;
 constexpr int kQCap = 32;             // repair jobs per warp and round
+constexpr int kMine = 4;              // jobs one thread queues per round
+constexpr int kAcc = 4;               // accumulator buffers in tensor memory
 constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
 constexpr float kU = 5.9604645e-08f;  // 2^-24
@@ -62,12 +64,12 @@ struct EncSmem {
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
     static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 8 warps x kQCap x 8 B
     static constexpr uint32_t misc = queue + 8 * kQCap * 8;
-    static constexpr uint32_t total = misc + 256;  // base is 1024-aligned (checked in-kernel)
+    static constexpr uint32_t total = misc + 320;  // base is 1024-aligned (checked in-kernel)
 };
 
 struct Misc {
     uint64_t full[kStages], empty[kStages];
-    uint64_t accfull[2], accempty[2];
+    uint64_t accfull[kAcc], accempty[kAcc];
     uint64_t gready[kSegBufs];
     uint64_t bfree;
     uint32_t tmem_slot;
@@ -75,6 +77,9 @@ struct Misc {
     int qcount[8];
     float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
 };
+
+static_assert(sizeof(Misc) <= 320, "Misc outgrew its shared-memory slot");
+static_assert(EncSmem::total <= 232448, "encode kernel exceeds 227 KB of shared memory");
 
 struct EncParams {
     RowArgs a;
@@ -99,6 +104,13 @@ template <typename T>
 __device__ __forceinline__ T pick4(const T (&v)[4], int i) {
     return i == 0 ? v[0] : i == 1 ? v[1] : i == 2 ? v[2] : v[3];
 }
+template <typename T>
+__device__ __forceinline__ void set4(T (&v)[4], int i, T x) {
+    v[0] = i == 0 ? x : v[0];
+    v[1] = i == 1 ? x : v[1];
+    v[2] = i == 2 ? x : v[2];
+    v[3] = i == 3 ? x : v[3];
+}
 
 // Rows of the gauge channels whose error bounds block bk's values: the whole gauge group
 // when the group spans the block, else the block's own channels.
@@ -113,28 +125,51 @@ __device__ __forceinline__ void bound_range(int bk, int g, int blk, int& lo, int
 }
 
 // Exact gauge-space value of (row, col) in the library's fixed order (pairwise sum of the
-// fp32 products), x read from the swizzled stage tile and G from global memory (fp32 row
-// `col` of the head's gauge set).
-__device__ __noinline__ float exact_z(const unsigned char* stage, int row, int col, const float* Gf, int g) {
+// fp32 products: 8-product trees merged with a binary carry), x read from the swizzled
+// stage tile and G from global memory (fp32 row `col` of the head's gauge set).
+__device__ __forceinline__ float exact_z(const unsigned char* stage, int row, int col, const float* Gf, int g) {
     const int r0 = (col / g) * g;
     const float* Grow = Gf + (size_t)col * g;
-    float s[16];
-#pragma unroll
-    for (int c = 0; c < 16; c++) {
-        s[c] = 0.0f;
-        if (c < g / 8) {
-            const int k = r0 + 8 * c;
-            const uint4 xv = *reinterpret_cast<const uint4*>(stage + (k >> 6) * 16384 + row * 128 +
-                                                             ((((k & 63) >> 3) ^ (row & 7)) << 4));
-            const float4 g0 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c));
-            const float4 g1 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c + 4));
-            const float ga[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-            const float xa[8] = {bf_lo(xv.x), bf_hi(xv.x), bf_lo(xv.y), bf_hi(xv.y),
-                                 bf_lo(xv.z), bf_hi(xv.z), bf_lo(xv.w), bf_hi(xv.w)};
-            s[c] = tree8(ga, xa);
+    float l0 = 0.0f, l1 = 0.0f, l2 = 0.0f, l3 = 0.0f, v = 0.0f;
+#pragma unroll 1
+    for (int c = 0; c < g / 8; c++) {
+        const int k = r0 + 8 * c;
+        const uint4 xv = *reinterpret_cast<const uint4*>(stage + (k >> 6) * 16384 + row * 128 +
+                                                         ((((k & 63) >> 3) ^ (row & 7)) << 4));
+        const float4 g0 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c));
+        const float4 g1 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c + 4));
+        const float ga[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+        const float xa[8] = {bf_lo(xv.x), bf_hi(xv.x), bf_lo(xv.y), bf_hi(xv.y),
+                             bf_lo(xv.z), bf_hi(xv.z), bf_lo(xv.w), bf_hi(xv.w)};
+        v = tree8(ga, xa);
+        if (c & 1) {
+            v = __fadd_rn(l0, v);
+            if (c & 2) {
+                v = __fadd_rn(l1, v);
+                if (c & 4) {
+                    v = __fadd_rn(l2, v);
+                    if (c & 8) v = __fadd_rn(l3, v);
+                    else l3 = v;
+                } else {
+                    l2 = v;
+                }
+            } else {
+                l1 = v;
+            }
+        } else {
+            l0 = v;
         }
     }
-    return tree_combine(s, g / 8);
+    return v;
+}
+
+// One warp-cooperative round: lanes compute the queued exact values (job word: row | col << 8).
+__device__ __noinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned char* stage, const float* Gf, int g,
+                                      int lane) {
+    for (int j = lane; j < nq; j += 32) {
+        const uint32_t jb = qjob[2 * j];
+        qjob[2 * j + 1] = __float_as_uint(exact_z(stage, (int)(jb & 0xffu), (int)((jb >> 8) & 0xffu), Gf, g));
+    }
 }
 
 __device__ __forceinline__ uint32_t scale16(float mx, float mn, float qmax) {
@@ -190,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             mbar_init(&M->full[i], 1);
             mbar_init(&M->empty[i], 4);
         }
-        for (int i = 0; i < 2; i++) {
+        for (int i = 0; i < kAcc; i++) {
             mbar_init(&M->accfull[i], 1);
             mbar_init(&M->accempty[i], 4);
         }
@@ -202,7 +237,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     for (uint32_t i = threadIdx.x; i < (uint32_t)npass * bsz / 16; i += kThreads)
         reinterpret_cast<uint4*>(bsplit)[i] = make_uint4(0, 0, 0, 0);
     if (warp == 1) {
-        tmem_alloc(&M->tmem_slot, 256);
+        tmem_alloc(&M->tmem_slot, kAcc * 128);
         tmem_relinquish();
         tc_fence_before();
     }
@@ -256,9 +291,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
                     cur = ti.seg;
                 }
-                const int st = i % kStages, buf = i & 1;
+                const int st = i % kStages, buf = i % kAcc;
                 ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
-                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i / kAcc) & 1) ^ 1, abort_flag, kWaitLimitNs);
                 if (!ok) {
                     *abort_flag = 1;
                     break;
@@ -287,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             if (*abort_flag && committed > 0) {
                 const int zero = 0;
                 const int i = committed - 1;
-                mbar_wait(&M->accfull[i & 1], (i >> 1) & 1, &zero, kWaitLimitNs);
+                mbar_wait(&M->accfull[i % kAcc], (i / kAcc) & 1, &zero, kWaitLimitNs);
             }
         }
     } else if (warp == 2) {
@@ -311,49 +346,68 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
             const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
-            float e_row[4];
+            {
+                // warm L2 with the next gauge set of this CTA (read at the next conversion)
+                int nl = ti.l, ns = ti.s, nh = ti.h + 1;
+                if (nh == a.H) {
+                    nh = 0;
+                    if (++ns == a.s_lo + a.s_n) {
+                        ns = a.s_lo;
+                        nl++;
+                    }
+                }
+                if (nl < a.L) {
+                    const char* nG = reinterpret_cast<const char*>(a.G + ((int64_t)(nl * 2 + ns) * a.H + nh) * (int64_t)kD * g);
+                    for (int off = lane * 128; off < kD * g * 4; off += 32 * 128)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(nG + off));
+                }
+            }
+            float e_row[4], s_g2[4], s_res2[4];
 #pragma unroll
-            for (int q = 0; q < 4; q++) {
-                const int n = lane + 32 * q;  // B row = output channel
-                const int r = n / g;
-                const float* Gr = Gf + (size_t)n * g;
-                float s_g2 = 0.0f, s_res2 = 0.0f;
-                for (int j = 0; j < g; j += 8) {
-                    const int k = r * g + j;
-                    const float4 v0 = __ldg(reinterpret_cast<const float4*>(Gr + j));
-                    const float4 v1 = __ldg(reinterpret_cast<const float4*>(Gr + j + 4));
-                    const float v[8] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w};
+            for (int q = 0; q < 4; q++) s_g2[q] = s_res2[q] = 0.0f;
+            for (int j = 0; j < g; j += 8) {
+                // the four rows of this lane: eight loads in flight per step
+                float4 v0[4], v1[4];
+#pragma unroll
+                for (int q = 0; q < 4; q++) {
+                    const float* Gr = Gf + (size_t)(lane + 32 * q) * g;
+                    v0[q] = __ldg(reinterpret_cast<const float4*>(Gr + j));
+                    v1[q] = __ldg(reinterpret_cast<const float4*>(Gr + j + 4));
+                }
+#pragma unroll
+                for (int q = 0; q < 4; q++) {
+                    const int n = lane + 32 * q;  // B row = output channel
+                    const int k = (n / g) * g + j;
+                    const float v[8] = {v0[q].x, v0[q].y, v0[q].z, v0[q].w, v1[q].x, v1[q].y, v1[q].z, v1[q].w};
                     uint32_t term[3][4];
 #pragma unroll
                     for (int e = 0; e < 8; e += 2) {
                         float rest0 = v[e], rest1 = v[e + 1];
-                        s_g2 = fmaf(v[e], v[e], s_g2);
-                        s_g2 = fmaf(v[e + 1], v[e + 1], s_g2);
+                        s_g2[q] = fmaf(v[e], v[e], s_g2[q]);
+                        s_g2[q] = fmaf(v[e + 1], v[e + 1], s_g2[q]);
 #pragma unroll
                         for (int t = 0; t < 3; t++) {
-                            if (t < npass) {
-                                const __nv_bfloat16 h0 = __float2bfloat16_rn(rest0);
-                                const __nv_bfloat16 h1 = __float2bfloat16_rn(rest1);
-                                rest0 = __fsub_rn(rest0, __bfloat162float(h0));
-                                rest1 = __fsub_rn(rest1, __bfloat162float(h1));
-                                term[t][e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) |
-                                                  ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-                            }
+                            const __nv_bfloat16 h0 = __float2bfloat16_rn(rest0);
+                            const __nv_bfloat16 h1 = __float2bfloat16_rn(rest1);
+                            rest0 = __fsub_rn(rest0, __bfloat162float(h0));
+                            rest1 = __fsub_rn(rest1, __bfloat162float(h1));
+                            term[t][e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) |
+                                              ((uint32_t)__bfloat16_as_ushort(h1) << 16);
                         }
-                        s_res2 = fmaf(rest0, rest0, s_res2);
-                        s_res2 = fmaf(rest1, rest1, s_res2);
+                        s_res2[q] = fmaf(rest0, rest0, s_res2[q]);
+                        s_res2[q] = fmaf(rest1, rest1, s_res2[q]);
                     }
 #pragma unroll
                     for (int t = 0; t < 3; t++) {
-                        if (t < npass) {
-                            unsigned char* region = bsplit + (npass - 1 - t) * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
-                            *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
-                                make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
-                        }
+                        unsigned char* region = bsplit + (npass - 1 - t) * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
+                        *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
+                            make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
                     }
                 }
-                e_row[q] = ((c_order + c_tc) * sqrtf(s_g2) + sqrtf(s_res2)) * 1.001f + 1e-30f;
             }
+#pragma unroll
+            for (int q = 0; q < 4; q++)
+                e_row[q] = ((c_order + c_tc) * sqrtf(s_g2[q]) + sqrtf(s_res2[q])) * 1.001f + 1e-30f;
             // per quantization block: max of e over the rows that bound its values
 #pragma unroll
             for (int bk = 0; bk < 4; bk++) {
@@ -378,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         }
     } else {
         // ------------------------------------------------------------ epilogue warpgroups
-        const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup = accumulator buffer
+        const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup: tiles i = wg (mod 2)
         const int q4 = warp & 3;                      // TMEM lane quadrant of this warp
         const int row = q4 * 32 + lane;               // tile row = TMEM lane
         const int qw = warp - kEpiWarp0;              // job queue of this warp
@@ -399,8 +453,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         for (int i = wg; i < my_tiles; i += 2, it.step(a, 2)) {
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
-            const int st = i % kStages, buf = wg;
-            bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+            const int st = i % kStages, buf = i % kAcc;
+            bool ok = mbar_wait(&M->accfull[buf], (i / kAcc) & 1, abort_flag, kWaitLimitNs);
             ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
             ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
             if (!__all_sync(0xffffffffu, ok)) {
@@ -415,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
             // ---- 1. ||x||^2 over the bound range of every block (bf16 -> fp32 exact)
             float bs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-#pragma unroll
+#pragma unroll 4
             for (int c8 = 0; c8 < 16; c8++) {
                 const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
                                                                  (((c8 & 7) ^ (row & 7)) << 4));
@@ -446,6 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             // ---- 2. approximate block ranges from the accumulator
             float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
             float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll 1
             for (int c = 0; c < 4; c++) {
                 uint32_t v[32];
                 tmem_ld32(tacc + c * 32, v);
@@ -459,12 +514,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 lo = fminf(lo, __uint_as_float(v[31]));
                 hi = fmaxf(hi, __uint_as_float(v[31]));
                 const int bk = (c * 32) / blk;
-#pragma unroll
-                for (int q = 0; q < 4; q++)
-                    if (q == bk) {
-                        mn[q] = fminf(mn[q], lo);
-                        mx[q] = fmaxf(mx[q], hi);
-                    }
+                set4(mn, bk, fminf(pick4(mn, bk), lo));
+                set4(mx, bk, fmaxf(pick4(mx, bk), hi));
             }
 
             // ---- 3. error bound per block; scale/zero from the intervals when they agree
@@ -490,14 +541,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
 
-            // ---- 4. exact extremes of ambiguous blocks (warp-cooperative)
+            // ---- 4. exact extremes of ambiguous blocks (warp-cooperative rounds)
             if (__any_sync(0xffffffffu, amb != 0)) {
-                float ex_mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
-                float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                int nmine = 0;
-                int ms[4] = {0, 0, 0, 0}, mt[4] = {0, 0, 0, 0};
-                if (lane == 0) M->qcount[qw] = 0;
-                __syncwarp();
+                // candidate masks per 32-column chunk: values within 2E of the block's min / max
+                uint32_t pm[4] = {0, 0, 0, 0}, px[4] = {0, 0, 0, 0};
+#pragma unroll 1
                 for (int c = 0; c < 4; c++) {
                     const int bk = (c * 32) / blk;
                     const int need = (amb >> (2 * bk)) & 3;
@@ -505,66 +553,62 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     uint32_t v[32];
                     tmem_ld32(tacc + c * 32, v);
                     tmem_wait_ld();
-                    if (!need) continue;
-                    const float e = pick4(E, bk);
-                    const float thr_lo = __fadd_rn(pick4(mn, bk), 2.0f * e);
-                    const float thr_hi = __fsub_rn(pick4(mx, bk), 2.0f * e);
-                    uint32_t mmin = 0, mmax = 0;
+                    const float e2 = 2.0f * pick4(E, bk);
+                    const float thr_lo = __fadd_rn(pick4(mn, bk), e2), thr_hi = __fsub_rn(pick4(mx, bk), e2);
+                    uint32_t a0 = 0, a1 = 0;
 #pragma unroll
                     for (int k = 0; k < 32; k++) {
                         const float z = __uint_as_float(v[k]);
-                        if (z <= thr_lo) mmin |= 1u << k;
-                        if (z >= thr_hi) mmax |= 1u << k;
+                        if (z <= thr_lo) a0 |= 1u << k;
+                        if (z >= thr_hi) a1 |= 1u << k;
                     }
-                    if (!(need & 1)) mmax = 0;
-                    uint32_t mall = mmin | mmax;
-                    while (mall) {
-                        const int k = __ffs(mall) - 1;
-                        mall &= mall - 1;
-                        const int tag = bk | (((mmin >> k) & 1) ? 4 : 0) | (((mmax >> k) & 1) ? 8 : 0);
-                        const int col = c * 32 + k;
-                        const int slot = atomicAdd(&M->qcount[qw], 1);
-                        if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
-                        if (slot < kQCap && nmine < 4) {
-#pragma unroll
-                            for (int m = 0; m < 4; m++)
-                                if (m == nmine) {
-                                    ms[m] = slot;
-                                    mt[m] = tag;
-                                }
-                            nmine++;
-                        } else {
-                            const float ze = exact_z(stg, row, col, Gf, g);
-#pragma unroll
-                            for (int q = 0; q < 4; q++)
-                                if (q == bk) {
-                                    if (tag & 4) ex_mn[q] = fminf(ex_mn[q], ze);
-                                    if (tag & 8) ex_mx[q] = fmaxf(ex_mx[q], ze);
-                                }
+                    set4(pm, c, need ? a0 : 0u);
+                    set4(px, c, (need & 1) ? a1 : 0u);
+                }
+                float ex_mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
+                float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                bool pend = (pm[0] | pm[1] | pm[2] | pm[3] | px[0] | px[1] | px[2] | px[3]) != 0;
+                while (__any_sync(0xffffffffu, pend)) {
+                    if (lane == 0) M->qcount[qw] = 0;
+                    __syncwarp();
+                    int sl[kMine] = {0, 0, 0, 0};
+                    uint32_t tg[kMine] = {0, 0, 0, 0};
+                    int nm = 0;
+#pragma unroll 1
+                    for (int c = 0; c < 4; c++) {
+                        uint32_t cm = pick4(pm, c), cx = pick4(px, c);
+                        while (nm < kMine && (cm | cx)) {
+                            const int k = __ffs(cm | cx) - 1;
+                            const uint32_t bit = 1u << k;
+                            const int slot = atomicAdd(&M->qcount[qw], 1);
+                            if (slot >= kQCap) break;
+                            const uint32_t col = (uint32_t)(c * 32 + k);
+                            const uint32_t tag = col | ((cm & bit) ? 0x100u : 0u) | ((cx & bit) ? 0x200u : 0u);
+                            qjob[2 * slot] = (uint32_t)row | (col << 8);
+                            set4(sl, nm, slot);
+                            set4(tg, nm, tag);
+                            nm++;
+                            cm &= ~bit;
+                            cx &= ~bit;
                         }
+                        set4(pm, c, cm);
+                        set4(px, c, cx);
                     }
-                }
-                __syncwarp();
-                const int nq = min(M->qcount[qw], kQCap);
-                for (int j = lane; j < nq; j += 32) {
-                    const uint32_t jb = qjob[2 * j];
-                    qjob[2 * j + 1] = __float_as_uint(exact_z(stg, (int)(jb & 0xffu), (int)(jb >> 8), Gf, g));
-                }
-                __syncwarp();
-#pragma unroll
-                for (int m = 0; m < 4; m++) {
-                    if (m < nmine) {
-                        const float ze = __uint_as_float(qjob[2 * ms[m] + 1]);
-                        const int tag = mt[m];
-#pragma unroll
-                        for (int q = 0; q < 4; q++)
-                            if (q == (tag & 3)) {
-                                if (tag & 4) ex_mn[q] = fminf(ex_mn[q], ze);
-                                if (tag & 8) ex_mx[q] = fmaxf(ex_mx[q], ze);
-                            }
+                    __syncwarp();
+                    const int nq = min(M->qcount[qw], kQCap);
+                    run_jobs(qjob, nq, stg, Gf, g, lane);
+                    __syncwarp();
+#pragma unroll 1
+                    for (int m = 0; m < nm; m++) {
+                        const uint32_t tgm = pick4(tg, m);
+                        const float ze = __uint_as_float(qjob[2 * pick4(sl, m) + 1]);
+                        const int bk = (int)(tgm & 0xffu) / blk;
+                        if (tgm & 0x100u) set4(ex_mn, bk, fminf(pick4(ex_mn, bk), ze));
+                        if (tgm & 0x200u) set4(ex_mx, bk, fmaxf(pick4(ex_mx, bk), ze));
                     }
+                    __syncwarp();
+                    pend = (pm[0] | pm[1] | pm[2] | pm[3] | px[0] | px[1] | px[2] | px[3]) != 0;
                 }
-                __syncwarp();
 #pragma unroll
                 for (int bk = 0; bk < 4; bk++) {
                     const int need = (amb >> (2 * bk)) & 3;
@@ -591,10 +635,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         const float cc = -mz * r;
                         rinv[bk] = r;
                         c0[bk] = cc;
-                        // |t~ - t|: the value bound E/s, plus the rounding of rcp, c0 and the fma
-                        // (a few ulps of |z r| + |c0|) and of the definition's subtract and divide
+                        // |t~ - t| <= E/s plus roundings: the fma and its inputs r and c0 (u|z r|,
+                        // 2u|c0|, u|t|) and the definition's subtract and divide (2u|t|)
                         const float zr = fmaxf(fabsf(mn[bk]), fabsf(mx[bk])) * r;
-                        const float mu = E[bk] * r * 1.0001f + (zr + fabsf(cc) + qmaxf + 1.0f) * 4.8e-7f;
+                        const float mu = E[bk] * r * 1.0001f + (zr + 2.0f * fabsf(cc) + 3.0f * (qmaxf + 1.0f)) * 6.6e-8f;
                         // mu < 1e-4: a code from z~ can only differ where the tolerance allows it
                         lim[bk] = mu < 0.99e-4f ? 2.0f : 0.5f - mu;
                         const float tlo = (mn[bk] - E[bk]) * r + cc, thi = (mx[bk] + E[bk]) * r + cc;
@@ -604,12 +648,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
 
-            // ---- 6. codes from z~, stored straight from registers; near-boundary values queued
+            // ---- 6. codes from z~, stored straight from registers; near-boundary values repaired
             uint8_t* crow = a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
-            int nmine = 0;
-            int ms[4] = {0, 0, 0, 0}, mt[4] = {0, 0, 0, 0};
-            if (lane == 0) M->qcount[qw] = 0;
-            __syncwarp();
+            uint32_t am[4] = {0, 0, 0, 0};  // values within mu of a rounding boundary
+#pragma unroll 1
             for (int c = 0; c < 4; c++) {
                 uint32_t v[32];
                 tmem_ld32(tacc + c * 32, v);
@@ -621,7 +663,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 uint32_t qv[32];
                 float dmax = 0.0f;
                 if (fst && lm > 1.0f) {
-                    // no value of this block can leave [0, qmax] and no boundary check is needed
 #pragma unroll
                     for (int k = 0; k < 32; k++) qv[k] = __float_as_uint(fmaf(__uint_as_float(v[k]), r, cc) + kMagic);
                 } else if (fst) {
@@ -667,55 +708,53 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     }
                 }
                 if (valid && lv && dmax > lm) {
-                    // rare: the values within the bound of a rounding boundary
-                    uint32_t amask = 0;
+                    uint32_t mk = 0;
 #pragma unroll
                     for (int k = 0; k < 32; k++) {
                         float t = fmaf(__uint_as_float(v[k]), r, cc);
                         if (!fst) t = fminf(fmaxf(t, 0.0f), qmaxf);
                         const float y = t + kMagic;
-                        if (fabsf(t - (y - kMagic)) > lm) amask |= 1u << k;
+                        if (fabsf(t - (y - kMagic)) > lm) mk |= 1u << k;
                     }
-                    while (amask) {
-                        const int k = __ffs(amask) - 1;
-                        amask &= amask - 1;
-                        const int col = c * 32 + k;
-                        const int slot = atomicAdd(&M->qcount[qw], 1);
-                        if (slot < kQCap) qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
-                        if (slot < kQCap && nmine < 4) {
-#pragma unroll
-                            for (int m = 0; m < 4; m++)
-                                if (m == nmine) {
-                                    ms[m] = slot;
-                                    mt[m] = col;
-                                }
-                            nmine++;
-                        } else {
-                            const float ze = exact_z(stg, row, col, Gf, g);
-                            const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
-                            patch_code<BITS>(crow, col * BITS, q);
-                        }
-                    }
+                    set4(am, c, mk);
                 }
             }
-            if (__any_sync(0xffffffffu, nmine > 0)) {
+            bool pend = (am[0] | am[1] | am[2] | am[3]) != 0;
+            while (__any_sync(0xffffffffu, pend)) {
+                if (lane == 0) M->qcount[qw] = 0;
+                __syncwarp();
+                int sl[kMine] = {0, 0, 0, 0}, cl[kMine] = {0, 0, 0, 0};
+                int nm = 0;
+#pragma unroll 1
+                for (int c = 0; c < 4; c++) {
+                    uint32_t ca = pick4(am, c);
+                    while (nm < kMine && ca) {
+                        const int k = __ffs(ca) - 1;
+                        const int slot = atomicAdd(&M->qcount[qw], 1);
+                        if (slot >= kQCap) break;
+                        const int col = c * 32 + k;
+                        qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
+                        set4(sl, nm, slot);
+                        set4(cl, nm, col);
+                        nm++;
+                        ca &= ca - 1;
+                    }
+                    set4(am, c, ca);
+                }
                 __syncwarp();
                 const int nq = min(M->qcount[qw], kQCap);
-                for (int j = lane; j < nq; j += 32) {
-                    const uint32_t jb = qjob[2 * j];
-                    qjob[2 * j + 1] = __float_as_uint(exact_z(stg, (int)(jb & 0xffu), (int)(jb >> 8), Gf, g));
+                run_jobs(qjob, nq, stg, Gf, g, lane);
+                __syncwarp();
+#pragma unroll 1
+                for (int m = 0; m < nm; m++) {
+                    const int col = pick4(cl, m);
+                    const float ze = __uint_as_float(qjob[2 * pick4(sl, m) + 1]);
+                    const int bk = col / blk;
+                    const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
+                    patch_code<BITS>(crow, col * BITS, q);
                 }
                 __syncwarp();
-#pragma unroll
-                for (int m = 0; m < 4; m++) {
-                    if (m < nmine) {
-                        const float ze = __uint_as_float(qjob[2 * ms[m] + 1]);
-                        const int col = mt[m];
-                        const int bk = col / blk;
-                        const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
-                        patch_code<BITS>(crow, col * BITS, q);
-                    }
-                }
+                pend = (am[0] | am[1] | am[2] | am[3]) != 0;
             }
 
             // ---- 7. scales; release the stage and the accumulator buffer
@@ -739,7 +778,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem, 256);
+        tmem_dealloc(tmem, kAcc * 128);
     }
 }
 
