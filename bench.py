@@ -153,6 +153,8 @@ def run_reference(args):
         return
     from paper_2607_20538_gb300 import synth
     w = synth.WORKLOADS[args.workload]
+    if args.layers:
+        w = w.replace(L=min(args.layers, w.L))
     G = synth.gauges(w)
     cores = os.cpu_count() or 1
     for _ in range(args.warmup):
@@ -189,6 +191,8 @@ def run_cuda(args):
         torch.cuda.set_device(0)
     dev = torch.cuda.current_device()
     w = synth.WORKLOADS[args.workload]
+    if args.layers:
+        w = w.replace(L=min(args.layers, w.L))
     shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
     nc, ns, nr = cg.packed_bytes(shape, params)
     x = synth.kv_cache(w, threads=max(4, (os.cpu_count() or 8) // max(ws, 1)))
@@ -321,6 +325,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
     ap.add_argument("--workload", default="llama3_8b")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="keep only the first N layers of the workload (small cases for profiling)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()

@@ -3,18 +3,21 @@
 //
 // Persistent warp-specialized kernel, one CTA per SM, 14 warps:
 //   warp 0      bulk-copy producer: the packed codes of a 128-token tile are contiguous
-//               (rows of 16*bits bytes); one cp.async.bulk per tile into a 4-stage ring;
+//               (rows of 16*bits bytes); one cp.async.bulk per tile into a ring of stages;
 //   warp 1      MMA issuer: D_k = A_k B^T on tcgen05, A = codes as bf16 (128 + q, exact),
 //               B = G^T of the gauge group split into two bf16 terms; one fp32
 //               accumulator per quantization sub-block k of a group (block < group gives
-//               two), double buffered in tensor memory;
+//               two), double buffered in tensor memory (tile i uses buffer i mod 2);
 //   warps 2..5  unpackers, one token row each: codes -> bf16 A tile (128-byte swizzle);
 //               at a gauge change they also build B and the per-column sums c_k[i] =
 //               sum_{j in sub-block k} G[j][i] of the split;
-//   warps 6..13 two epilogue warpgroups; warpgroup k owns accumulator buffer k and takes
-//               every other tile; one token row (TMEM lane) per thread:
-//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i], bf16 store. Each
-//               thread loads its next tile's block scales one tile ahead.
+//   warps 6..13 epilogue: both warpgroups work on every tile, warpgroup h on output
+//               columns 64h..64h+63, one token row (TMEM lane) per thread:
+//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i]. The accumulator
+//               buffer is released as soon as it is in registers, so the MMAs of tile i+2
+//               overlap the arithmetic of tile i; each warp stages its 32 x 64 bf16 block
+//               in shared memory (128-byte swizzle) and writes it with one TMA tile store.
+//               Each thread loads the next tile's block scales one tile ahead.
 // With the scale and zero of a block constant along the token, dequantization commutes
 // with the rotation, so the integer codes go through the tensor cores unscaled.
 #include <cuda_bf16.h>
@@ -22,6 +25,7 @@
 #include "cg_sm100.cuh"
 #include "cg_tc.h"
 #include "cg_tc_common.cuh"
+#include "cg_tmap.h"
 
 namespace cg {
 namespace {
@@ -32,29 +36,39 @@ using tc::kWaitLimitNs;
 
 constexpr int kThreads = 448;
 constexpr int kEpiWarp0 = 6;
-constexpr int kCStages = 4;
-constexpr int kCStageBytes = 128 * 128;  // up to 8-bit codes: 128 rows x 128 B
 constexpr int kATile = 128 * kD * 2;
 constexpr int kSegBufs = 4;
+constexpr int kMaxCStages = 4;
+constexpr uint32_t kOutWarpBytes = 32 * 128;  // 32 rows x 64 bf16 per epilogue warp
+constexpr int kMmaPerTile = 16;  // 2 split terms x 128 / 16 K steps, for every group and block
 
+template <int BITS>
 struct DecSmem {
-    static constexpr uint32_t a_tiles = 0;                          // 2 x 32 KB
-    static constexpr uint32_t bsplit = a_tiles + 2 * kATile;        // 2 x (16 or 32 KB)
-    static constexpr uint32_t cstages = bsplit + 2 * 32768;         // 4 x 16 KB
-    static constexpr uint32_t csum = cstages + kCStages * kCStageBytes;  // [4][2][128] fp32
+    static constexpr int cstages_n = BITS == 8 ? 3 : 4;
+    static constexpr uint32_t cstage_bytes = 128u * 16u * BITS;  // 128 rows of packed codes
+    static constexpr uint32_t a_tiles = 0;                        // 2 x 32 KB
+    static constexpr uint32_t bsplit = a_tiles + 2 * kATile;      // 2 x (16 or 32 KB)
+    static constexpr uint32_t ostage = bsplit + 2 * 32768;        // 8 warps x 4 KB
+    static constexpr uint32_t cstages = ostage + 8 * kOutWarpBytes;
+    static constexpr uint32_t csum = cstages + cstages_n * cstage_bytes;  // [4][2][128] fp32
     static constexpr uint32_t misc = csum + kSegBufs * 2 * kD * 4;
     static constexpr uint32_t total = misc + 512;
+    static_assert(ostage % 1024 == 0 && cstages % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+    static_assert(total + 1024 <= 232448, "shared memory budget");
 };
 
 struct DecMisc {
-    uint64_t cfull[kCStages], cempty[kCStages];
+    uint64_t cfull[kMaxCStages], cempty[kMaxCStages];
     uint64_t afull[2], aempty[2];
     uint64_t accfull[2], accempty[2];
     uint64_t gready[kSegBufs];
     uint64_t bfree;
+    uint32_t mseq[16][4];  // the MMA sequence of a tile
     uint32_t tmem_slot;
     int abort_flag;
 };
+
+static_assert(sizeof(DecMisc) <= 512, "misc block");
 
 struct DecParams {
     RowArgs a;
@@ -65,41 +79,59 @@ struct DecParams {
 // codes of one row (128 codes, little-endian bit stream) -> 16 chunks of 8 bf16 (128 + q)
 template <int BITS>
 __device__ __forceinline__ void unpack_row(const uint32_t* w, uint4 (&out)[16]) {
+    if constexpr (BITS == 4) {
+        // eight nibbles per word: split low/high nibbles, interleave them back into code
+        // order with byte permutes, then pair each code byte with the 0x43 exponent byte
 #pragma unroll
-    for (int c = 0; c < 16; c++) {
-        uint32_t o[4];
-#pragma unroll
-        for (int e = 0; e < 4; e++) {
-            uint32_t q[2];
-#pragma unroll
-            for (int h = 0; h < 2; h++) {
-                const int k = 8 * c + 2 * e + h;
-                const int p = k * BITS;
-                uint32_t v = w[p >> 5] >> (p & 31);
-                if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
-                q[h] = v & ((1u << BITS) - 1u);
-            }
-            if (BITS < 8) {
-                o[e] = 0x43004300u | q[0] | (q[1] << 16);
-            } else {
-                const __nv_bfloat162 b2 = __floats2bfloat162_rn((float)q[0], (float)q[1]);
-                o[e] = *reinterpret_cast<const uint32_t*>(&b2);
-            }
+        for (int c = 0; c < 16; c++) {
+            const uint32_t lo_n = w[c] & 0x0F0F0F0Fu;         // codes 0, 2, 4, 6 of the word
+            const uint32_t hi_n = (w[c] >> 4) & 0x0F0F0F0Fu;  // codes 1, 3, 5, 7
+            const uint32_t q03 = __byte_perm(lo_n, hi_n, 0x5140);  // codes 0..3 as bytes
+            const uint32_t q47 = __byte_perm(lo_n, hi_n, 0x7362);  // codes 4..7
+            out[c] = make_uint4(__byte_perm(q03, 0x43u, 0x4140), __byte_perm(q03, 0x43u, 0x4342),
+                                __byte_perm(q47, 0x43u, 0x4140), __byte_perm(q47, 0x43u, 0x4342));
         }
-        out[c] = make_uint4(o[0], o[1], o[2], o[3]);
+    } else {
+#pragma unroll
+        for (int c = 0; c < 16; c++) {
+            uint32_t o[4];
+#pragma unroll
+            for (int e = 0; e < 4; e++) {
+                uint32_t q[2];
+#pragma unroll
+                for (int h = 0; h < 2; h++) {
+                    const int k = 8 * c + 2 * e + h;
+                    const int p = k * BITS;
+                    uint32_t v = w[p >> 5] >> (p & 31);
+                    if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
+                    q[h] = v & ((1u << BITS) - 1u);
+                }
+                if (BITS < 8) {
+                    o[e] = 0x43004300u | q[0] | (q[1] << 16);
+                } else {
+                    const __nv_bfloat162 b2 = __floats2bfloat162_rn((float)q[0], (float)q[1]);
+                    o[e] = *reinterpret_cast<const uint32_t*>(&b2);
+                }
+            }
+            out[c] = make_uint4(o[0], o[1], o[2], o[3]);
+        }
     }
 }
 
 template <int BITS>
-__global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams P) {
+__global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_constant__ CUtensorMap omap,
+                                                                 const DecParams P) {
+    using SL = DecSmem<BITS>;
+    constexpr int kCStages = SL::cstages_n;
+    constexpr uint32_t kCStageBytes = SL::cstage_bytes;
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const uint32_t base_u32 = (smem_u32(smem_raw) + 1023u) & ~1023u;
     unsigned char* sm = smem_raw + (base_u32 - smem_u32(smem_raw));
-    DecMisc* M = reinterpret_cast<DecMisc*>(sm + DecSmem::misc);
-    unsigned char* atiles = sm + DecSmem::a_tiles;
-    unsigned char* bsplit = sm + DecSmem::bsplit;
-    unsigned char* cst = sm + DecSmem::cstages;
-    float* csum = reinterpret_cast<float*>(sm + DecSmem::csum);
+    DecMisc* M = reinterpret_cast<DecMisc*>(sm + SL::misc);
+    unsigned char* atiles = sm + SL::a_tiles;
+    unsigned char* bsplit = sm + SL::bsplit;
+    unsigned char* cst = sm + SL::cstages;
+    float* csum = reinterpret_cast<float*>(sm + SL::csum);
 
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
@@ -125,7 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             mbar_init(&M->afull[i], 4);
             mbar_init(&M->aempty[i], 1);
             mbar_init(&M->accfull[i], 1);
-            mbar_init(&M->accempty[i], 4);
+            mbar_init(&M->accempty[i], 8);
         }
         for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 4);
         mbar_init(&M->bfree, 1);
@@ -175,11 +207,42 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && my_tiles > 0) {
             const uint32_t idesc = idesc_bf16_f32(128, gb);
+            // The MMAs of a tile form a fixed sequence (16 for every supported group and
+            // block): D column offset, A and B byte offsets, accumulate flag. It is laid out
+            // once; per tile only the stage bases change.
+            int nseq = 0;
+            {
+                int& n = nseq;
+                for (int p = 0; p < 2; p++)
+                    for (int r = 0; r < 128 / gb; r++)
+                        for (int k = 0; k < nsub; k++) {
+                            const int kw = nsub > 1 ? blk : gb;  // K width of this sub-block
+                            const int kbeg = r * gb + k * (nsub > 1 ? blk : 0);
+                            for (int ks = 0; ks < kw / 16 && n < kMmaPerTile; ks++, n++) {
+                                const int k0 = kbeg + ks * 16;
+                                M->mseq[n][0] = (uint32_t)(k * 128 + r * gb);
+                                M->mseq[n][1] = (uint32_t)((k0 >> 6) * 16384 + (k0 & 63) * 2);
+                                M->mseq[n][2] = (uint32_t)(p * bsz + (g == 128 ? (k0 >> 6) * 16384 : 0) +
+                                                           (r * gb) * 128 + (k0 & 63) * 2);
+                                M->mseq[n][3] = (p > 0 || ks > 0) ? 1u : 0u;
+                            }
+                        }
+            }
+            uint32_t q_d[kMmaPerTile], q_a[kMmaPerTile], q_b[kMmaPerTile], q_acc = 0;
+#pragma unroll
+            for (int q = 0; q < kMmaPerTile; q++) {
+                q_d[q] = M->mseq[q][0];
+                q_a[q] = M->mseq[q][1] >> 4;
+                q_b[q] = M->mseq[q][2] >> 4;
+                q_acc |= M->mseq[q][3] << q;
+            }
+            const uint64_t bdesc = sdesc_sw128(smem_u32(bsplit));
             int64_t cur = -1;
             int committed = 0;
             tc::TileIter it;
             it.init(a, S, t_begin);
-            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            if (nseq != kMmaPerTile) *abort_flag = 1;  // unreachable for the eligible shapes
+            for (int i = 0; i < my_tiles && nseq == kMmaPerTile; i++, it.step(a, 1)) {
                 const tc::TileInfo ti = it.info(a);
                 const int64_t ls = ti.seg - seg0;
                 bool ok = true;
@@ -195,25 +258,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                     break;
                 }
                 tc_fence_after();
-                const uint32_t a_base = smem_u32(atiles + ab * kATile);
+                const uint64_t adesc = sdesc_sw128(smem_u32(atiles + ab * kATile));
                 const uint32_t d_base = tmem + buf * acc_cols;
-                for (int p = 0; p < 2; p++) {
-                    const uint32_t b_base = smem_u32(bsplit) + p * bsz;
-                    for (int r = 0; r < 128 / gb; r++) {
-                        for (int k = 0; k < nsub; k++) {
-                            const int kw = nsub > 1 ? blk : gb;           // K width of this sub-block
-                            const int kbeg = r * gb + k * (nsub > 1 ? blk : 0);
-                            for (int ks = 0; ks < kw / 16; ks++) {
-                                const int k0 = kbeg + ks * 16;
-                                const uint32_t a_addr = a_base + (k0 >> 6) * 16384 + (k0 & 63) * 2;
-                                const uint32_t b_addr =
-                                    b_base + (g == 128 ? (k0 >> 6) * 16384 : 0) + (r * gb) * 128 + (k0 & 63) * 2;
-                                mma_bf16(d_base + k * 128 + r * gb, sdesc_sw128(a_addr), sdesc_sw128(b_addr), idesc,
-                                         (p > 0 || ks > 0) ? 1u : 0u);
-                            }
-                        }
-                    }
-                }
+#pragma unroll
+                for (int q = 0; q < kMmaPerTile; q++)
+                    mma_bf16(d_base + q_d[q], adesc + q_a[q], bdesc + q_b[q], idesc, (q_acc >> q) & 1u);
                 mma_commit(&M->accfull[buf]);
                 mma_commit(&M->aempty[ab]);
                 const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
@@ -249,7 +298,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                 // B[n][k] = G_r[k - r g][n - r g]: thread `row` builds output channel n = row
                 const int n = row, r = n / g, i_in = n - r * g;
                 const float* Gc = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g + (int64_t)r * g * g + i_in;
-                float cs[2] = {0.0f, 0.0f};
+                float cs0 = 0.0f, cs1 = 0.0f;
                 for (int j = 0; j < g; j += 8) {
                     uint32_t hi[4], lo[4];
 #pragma unroll
@@ -263,8 +312,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                         lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
                         const float t2 = (__bfloat162float(h0) + __bfloat162float(l0)) +
                                          (__bfloat162float(h1) + __bfloat162float(l1));
-                        const int ksub = (nsub > 1 && j + e >= blk) ? 1 : 0;
-                        cs[ksub] += t2;
+                        if (nsub > 1 && j + e >= blk) cs1 += t2;
+                        else cs0 += t2;
                     }
                     const int k = r * g + j;
                     unsigned char* reg1 = bsplit + 1 * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
@@ -273,8 +322,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                     *reinterpret_cast<uint4*>(reg0 + sw128_offset(n, k & 63)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                 }
                 float* cb = csum + (ls & 3) * 2 * kD;
-                cb[n] = cs[0];
-                cb[kD + n] = cs[1];
+                cb[n] = cs0;
+                cb[kD + n] = cs1;
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
@@ -313,13 +362,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             }
         }
     } else {
-        // ------------------------------------------------------------ epilogue warpgroups
-        const int wg = (warp - kEpiWarp0) >> 2;  // warpgroup = accumulator buffer
-        const int ew = warp & 3;
-        const int row = ew * 32 + lane;
+        // ------------------------------------------------------------ epilogue
+        const int ew = warp - kEpiWarp0;  // 0..7
+        const int half = ew >> 2;         // output columns 64*half .. 64*half + 63
+        const int q4 = warp & 3;          // TMEM lane quadrant of this warp
+        const int row = q4 * 32 + lane;
         const int nbk = kD / blk;
+        unsigned char* ost = sm + SL::ostage + ew * kOutWarpBytes;
         tc::TileIter it;
-        it.init(a, S, t_begin + wg);
+        it.init(a, S, t_begin);
         // block scales of this thread's row, loaded one tile ahead
         uint32_t sz_next[4] = {0, 0, 0, 0};
         auto load_scales = [&](const tc::TileInfo& t, uint32_t (&dst)[4]) {
@@ -330,17 +381,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                     if (bk < nbk) dst[bk] = __ldg(sp + bk);
             }
         };
-        if (wg < my_tiles) load_scales(it.info(a), sz_next);
-        for (int i = wg; i < my_tiles; i += 2, it.step(a, 2)) {
+        if (my_tiles > 0) load_scales(it.info(a), sz_next);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
-            const int buf = wg;
+            const int buf = i & 1;
             uint32_t sz[4];
 #pragma unroll
             for (int q = 0; q < 4; q++) sz[q] = sz_next[q];
-            if (i + 2 < my_tiles) {
+            if (i + 1 < my_tiles) {
                 tc::TileIter nx = it;
-                nx.step(a, 2);
+                nx.step(a, 1);
                 load_scales(nx.info(a), sz_next);
             }
             bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
@@ -351,12 +402,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
             }
             tc_fence_after();
             const bool valid = row < ti.rows_valid;
+            // the warp's 32 rows all exist: staged and written by one TMA store; else the
+            // valid rows are stored directly
+            const bool whole = q4 * 32 + 32 <= ti.rows_valid;
             const float* cb = csum + (ls & 3) * 2 * kD;
-            const uint32_t tacc = tmem + ((uint32_t)(ew * 32) << 16) + buf * acc_cols;
-            uint4* orow = reinterpret_cast<uint4*>(a.out + (tc::dense_row(a, ti) + row) * kD);
+            const uint32_t tacc = tmem + ((uint32_t)(q4 * 32) << 16) + buf * acc_cols;
+            const int64_t row0 = tc::dense_row(a, ti) + q4 * 32;  // first row of this warp
+            uint4* orow = reinterpret_cast<uint4*>(a.out + (row0 + lane) * kD);
+            // the previous TMA store of this warp has finished reading the staging block
+            if (lane == 0) bulk_wait_read<0>();
+            __syncwarp();
 #pragma unroll
-            for (int c = 0; c < 4; c++) {
-                // chunk c: columns 32c..32c+31; gauge group r = 32c / g (g >= 32) or several (g < 32)
+            for (int cc = 0; cc < 2; cc++) {
+                const int c = 2 * half + cc;  // 32-column chunk of the tile
+                // gauge group r = 32c / g (g >= 32) or several (g < 32, then nsub = 1)
                 const int r = (c * 32) / g;
                 float sk[2], ak[2];
 #pragma unroll
@@ -375,29 +434,56 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
                 tmem_ld32(tacc + c * 32, d0);
                 if (nsub > 1) tmem_ld32(tacc + 128 + c * 32, d1);
                 tmem_wait_ld();
+                if (cc == 1) {
+                    // everything this warp needs from the buffer is in registers
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&M->accempty[buf]);
+                }
                 uint32_t o[16];
 #pragma unroll
-                for (int e = 0; e < 32; e += 2) {
-                    float x2[2];
-#pragma unroll
-                    for (int hh = 0; hh < 2; hh++) {
-                        const int col = c * 32 + e + hh;
-                        float xv = fmaf(sk[0], __uint_as_float(d0[e + hh]), ak[0] * cb[col]);
-                        if (nsub > 1) xv = fmaf(sk[1], __uint_as_float(d1[e + hh]), fmaf(ak[1], cb[kD + col], xv));
-                        x2[hh] = xv;
+                for (int e = 0; e < 32; e += 4) {
+                    const float4 c0 = *reinterpret_cast<const float4*>(cb + c * 32 + e);
+                    float x4[4] = {fmaf(sk[0], __uint_as_float(d0[e]), ak[0] * c0.x),
+                                   fmaf(sk[0], __uint_as_float(d0[e + 1]), ak[0] * c0.y),
+                                   fmaf(sk[0], __uint_as_float(d0[e + 2]), ak[0] * c0.z),
+                                   fmaf(sk[0], __uint_as_float(d0[e + 3]), ak[0] * c0.w)};
+                    if (nsub > 1) {
+                        const float4 c1 = *reinterpret_cast<const float4*>(cb + kD + c * 32 + e);
+                        x4[0] = fmaf(sk[1], __uint_as_float(d1[e]), fmaf(ak[1], c1.x, x4[0]));
+                        x4[1] = fmaf(sk[1], __uint_as_float(d1[e + 1]), fmaf(ak[1], c1.y, x4[1]));
+                        x4[2] = fmaf(sk[1], __uint_as_float(d1[e + 2]), fmaf(ak[1], c1.z, x4[2]));
+                        x4[3] = fmaf(sk[1], __uint_as_float(d1[e + 3]), fmaf(ak[1], c1.w, x4[3]));
                     }
-                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(x2[0], x2[1]);
-                    o[e >> 1] = *reinterpret_cast<const uint32_t*>(&b2);
+                    const __nv_bfloat162 b0 = __floats2bfloat162_rn(x4[0], x4[1]);
+                    const __nv_bfloat162 b1 = __floats2bfloat162_rn(x4[2], x4[3]);
+                    o[e >> 1] = *reinterpret_cast<const uint32_t*>(&b0);
+                    o[(e >> 1) + 1] = *reinterpret_cast<const uint32_t*>(&b1);
                 }
-                if (valid) {
+                if (whole) {
+                    // row `lane` of the warp's 32 x 128 B block; 16-byte unit u at u ^ (lane & 7)
 #pragma unroll
-                    for (int q = 0; q < 4; q++) orow[c * 4 + q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                    for (int q = 0; q < 4; q++) {
+                        const int u = cc * 4 + q;
+                        *reinterpret_cast<uint4*>(ost + lane * 128 + ((u ^ (lane & 7)) << 4)) =
+                            make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                    }
+                } else if (valid) {
+#pragma unroll
+                    for (int q = 0; q < 4; q++)
+                        orow[c * 4 + q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&M->accempty[buf]);
+            if (whole) {
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_2d(&omap, ost, 64 * half, (int)row0);
+                    bulk_commit();
+                }
+            }
         }
+        if (lane == 0) bulk_wait<0>();
     }
     __syncthreads();
     if (*abort_flag && threadIdx.x == 0) raise_flag(a.status, CG_FLAG_PIPE_TIMEOUT);
@@ -409,12 +495,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const DecParams 
 }
 
 template <int BITS>
-cudaError_t launch_dec(const DecParams& P, cudaStream_t st) {
-    const size_t smem = DecSmem::total + 1024;
+cudaError_t launch_dec(const DecParams& P, const CUtensorMap& omap, cudaStream_t st) {
+    const size_t smem = DecSmem<BITS>::total + 1024;
     cudaError_t e = cudaFuncSetAttribute(tc_decode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
-    tc_decode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(P);
+    tc_decode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(omap, P);
     return cudaGetLastError();
 }
 
@@ -426,7 +512,9 @@ bool tc_row_decode_eligible(const RowArgs& a) {
     if (a.blk < a.g && a.g / a.blk > 2) return false;
     if (a.t_count < 64) return false;
     if ((reinterpret_cast<uintptr_t>(a.codes) & 15u) || (reinterpret_cast<uintptr_t>(a.out) & 15u)) return false;
-    return true;
+    const int64_t rows = (int64_t)a.L * 2 * a.B * a.H * a.T_x;
+    if (rows + 128 >= (int64_t)1 << 31) return false;
+    return tmap_encode_fn() != nullptr;
 }
 
 cudaError_t tc_launch_row_decode(const RowArgs& a, cudaStream_t st) {
@@ -435,12 +523,16 @@ cudaError_t tc_launch_row_decode(const RowArgs& a, cudaStream_t st) {
     P.S = tc::make_sched(a);
     P.nsub = a.blk < a.g ? a.g / a.blk : 1;
     if (P.S.n_tiles == 0) return cudaSuccess;
+    // output rows [L][2][B][H][T_x] of 128 bf16, written in 32-row x 64-column boxes
+    CUtensorMap omap;
+    const uint64_t rows = (uint64_t)a.L * 2 * a.B * a.H * a.T_x;
+    if (!make_tmap_bf16_sw128(&omap, a.out, rows, kD, kD * 2, 32)) return cudaErrorInvalidValue;
     switch (a.bits) {
-        case 2: return launch_dec<2>(P, st);
-        case 3: return launch_dec<3>(P, st);
-        case 4: return launch_dec<4>(P, st);
-        case 6: return launch_dec<6>(P, st);
-        case 8: return launch_dec<8>(P, st);
+        case 2: return launch_dec<2>(P, omap, st);
+        case 3: return launch_dec<3>(P, omap, st);
+        case 4: return launch_dec<4>(P, omap, st);
+        case 6: return launch_dec<6>(P, omap, st);
+        case 8: return launch_dec<8>(P, omap, st);
         default: return cudaErrorInvalidValue;
     }
 }
