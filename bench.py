@@ -43,6 +43,22 @@ def _peaks():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def rank_reduce(v: float, op: str, device=None) -> float:
+    """Max or min of a per-rank scalar over the job (identity without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return v
+    t = torch.tensor([v], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX if op == "max" else dist.ReduceOp.MIN)
+    return float(t.item())
+
+
+def job_throughput(bytes_per_rank_step: int, world: int, ms_per_step: float) -> float:
+    """Whole-job GB/s: every rank processes its own shard of the same size (weak scaling)."""
+    return world * bytes_per_rank_step / (ms_per_step * 1e-3) / 1e9
+
+
 def _dist():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -240,12 +256,9 @@ def run_cuda(args):
     total_ms = t_start.elapsed_time(t_end)
     enc_ms = [e[0].elapsed_time(e[1]) for e in evs]
     dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    if ws > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = rank_reduce(total_ms, "max", dev)
     ms_step = total_ms / args.steps
-    value = ws * 2 * n_bf16 / (ms_step * 1e-3) / 1e9
+    value = job_throughput(2 * n_bf16, ws, ms_step)
     enc_avg, dec_avg = statistics.mean(enc_ms), statistics.mean(dec_ms)
     enc_alg = n_bf16 + nc + ns + nr + g_bytes
     dec_alg = nc + ns + nr + g_bytes + n_bf16
@@ -277,12 +290,8 @@ def run_cuda(args):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    e2e_val = ws * 2 * n_bf16 / (e2e_ms * 1e-3) / 1e9
-    if ws > 1:
-        t = torch.tensor([e2e_val], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MIN)
-        e2e_val = float(t.item()) * 1.0
+    e2e_ms = rank_reduce(e0.elapsed_time(e1) / e2e_steps, "max", dev)
+    e2e_val = job_throughput(2 * n_bf16, ws, e2e_ms)
     flags = cg.get_status()
     if flags:
         raise RuntimeError(f"device status flags {flags} after the timed region")
