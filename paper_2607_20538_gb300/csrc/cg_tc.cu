@@ -31,8 +31,8 @@
 // The accepted tolerance lets a code differ by one where t lies within 1e-4 steps of a
 // boundary, so blocks with mu < 1e-4 keep the z~ codes; in blocks with a larger mu the
 // codes within mu of a boundary are recomputed exactly. Recomputation uses the library's
-// order (as the CUDA-core kernels do), spread over the lanes of a warp by a shared-memory
-// job queue.
+// order (as the CUDA-core kernels do): candidates go into a per-warp shared-memory job
+// queue and teams of lanes compute them together.
 #include <cuda_bf16.h>
 
 #include "cg_sm100.cuh"
@@ -124,51 +124,49 @@ __device__ __forceinline__ void bound_range(int bk, int g, int blk, int& lo, int
     }
 }
 
-// Exact gauge-space value of (row, col) in the library's fixed order (pairwise sum of the
-// fp32 products: 8-product trees merged with a binary carry), x read from the swizzled
-// stage tile and G from global memory (fp32 row `col` of the head's gauge set).
-__device__ __forceinline__ float exact_z(const unsigned char* stage, int row, int col, const float* Gf, int g) {
-    const int r0 = (col / g) * g;
-    const float* Grow = Gf + (size_t)col * g;
-    float l0 = 0.0f, l1 = 0.0f, l2 = 0.0f, l3 = 0.0f, v = 0.0f;
-#pragma unroll 1
-    for (int c = 0; c < g / 8; c++) {
-        const int k = r0 + 8 * c;
-        const uint4 xv = *reinterpret_cast<const uint4*>(stage + (k >> 6) * 16384 + row * 128 +
-                                                         ((((k & 63) >> 3) ^ (row & 7)) << 4));
-        const float4 g0 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c));
-        const float4 g1 = __ldg(reinterpret_cast<const float4*>(Grow + 8 * c + 4));
-        const float ga[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-        const float xa[8] = {bf_lo(xv.x), bf_hi(xv.x), bf_lo(xv.y), bf_hi(xv.y),
-                             bf_lo(xv.z), bf_hi(xv.z), bf_lo(xv.w), bf_hi(xv.w)};
-        v = tree8(ga, xa);
-        if (c & 1) {
-            v = __fadd_rn(l0, v);
-            if (c & 2) {
-                v = __fadd_rn(l1, v);
-                if (c & 4) {
-                    v = __fadd_rn(l2, v);
-                    if (c & 8) v = __fadd_rn(l3, v);
-                    else l3 = v;
-                } else {
-                    l2 = v;
-                }
-            } else {
-                l1 = v;
-            }
-        } else {
-            l0 = v;
-        }
-    }
-    return v;
-}
-
-// One warp-cooperative round: lanes compute the queued exact values (job word: row | col << 8).
+// One warp-wide round of exact recomputation of the queued gauge-space values (job word:
+// row | col << 8; the value goes to the next word), in the library's fixed order. A team
+// of T = g/4 lanes computes one value: lane j forms the products of channels 4j..4j+3 and
+// their pairwise sum, and the team combines its partial sums with xor-shuffles, which
+// follows the same pairwise tree. Each lane loads the operands of kSlots values before any
+// arithmetic, so one memory round trip serves kSlots x (32 / T) values.
+constexpr int kSlots = 4;
 __device__ __noinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned char* stage, const float* Gf, int g,
                                       int lane) {
-    for (int j = lane; j < nq; j += 32) {
-        const uint32_t jb = qjob[2 * j];
-        qjob[2 * j + 1] = __float_as_uint(exact_z(stage, (int)(jb & 0xffu), (int)((jb >> 8) & 0xffu), Gf, g));
+    const int lgT = 29 - __clz(g);  // log2(g / 4); g in {8, ..., 128}
+    const int T = 1 << lgT, teams = 32 >> lgT;
+    const int tm = lane >> lgT, j = lane & (T - 1);
+    for (int base = 0; base < nq; base += kSlots * teams) {
+        uint2 xv[kSlots];
+        float4 gv[kSlots];
+#pragma unroll
+        for (int k = 0; k < kSlots; k++) {
+            const int c = base + k * teams + tm;
+            const uint32_t jb = qjob[2 * (c < nq ? c : 0)];
+            const int row = (int)(jb & 0xffu), col = (int)((jb >> 8) & 0xffu);
+            const int kk = (col & ~(g - 1)) + 4 * j;  // first channel of this lane's products
+            xv[k] = *reinterpret_cast<const uint2*>(stage + (kk >> 6) * 16384 + row * 128 +
+                                                    ((((kk & 63) >> 3) ^ (row & 7)) << 4) + (kk & 7) * 2);
+            gv[k] = __ldg(reinterpret_cast<const float4*>(Gf + (size_t)col * g + 4 * j));
+        }
+        float part[kSlots];
+#pragma unroll
+        for (int k = 0; k < kSlots; k++) {
+            const float p0 = __fmul_rn(gv[k].x, bf_lo(xv[k].x)), p1 = __fmul_rn(gv[k].y, bf_hi(xv[k].x));
+            const float p2 = __fmul_rn(gv[k].z, bf_lo(xv[k].y)), p3 = __fmul_rn(gv[k].w, bf_hi(xv[k].y));
+            part[k] = __fadd_rn(__fadd_rn(p0, p1), __fadd_rn(p2, p3));
+        }
+        for (int w = 1; w < T; w <<= 1) {
+#pragma unroll
+            for (int k = 0; k < kSlots; k++) part[k] = __fadd_rn(part[k], __shfl_xor_sync(0xffffffffu, part[k], w));
+        }
+        if (j == 0) {
+#pragma unroll
+            for (int k = 0; k < kSlots; k++) {
+                const int c = base + k * teams + tm;
+                if (c < nq) qjob[2 * c + 1] = __float_as_uint(part[k]);
+            }
+        }
     }
 }
 
