@@ -146,6 +146,20 @@ def kv_cache(w: Workload, T: int | None = None, threads: int = 8) -> np.ndarray:
     return out
 
 
+def rolling_history_layer(w: Workload, threads: int = 8) -> np.ndarray:
+    """History tokens [0, T_cap - 1) of the rolling workload for ONE layer, [1][2][B][H][T_cap-1][d].
+
+    Every layer's history is this one draw (layer 0's units); the per-layer gauges still
+    differ. A full independent draw of the 32-layer, batch-64, 16k-token history is 137 GB
+    of bf16, too much to generate on the host for a test or a benchmark."""
+    return kv_cache(w.replace(L=1, T=w.T_cap - 1), threads=threads)
+
+
+def rolling_new_token(w: Workload, threads: int = 8) -> np.ndarray:
+    """The token appended at position T_cap - 1 of every sequence, [L][2][B][H][1][d] (its own seed)."""
+    return kv_cache(w.replace(T=1, kv_seed=w.kv_seed + 500), threads=threads)
+
+
 def random_orthogonal(g: int, rng: np.random.Generator) -> np.ndarray:
     a = rng.standard_normal((g, g))
     q, r = np.linalg.qr(a)
