@@ -154,6 +154,25 @@ void bu_maps(const cg_shape* sh, const Sizes& z, int64_t rowbytes, int64_t rowsc
     sm->base = (int64_t)sh->t0 * rowscales;
 }
 
+// Row map for KIVI keys seen as rows of the key tensor: codes [B][H][n_q/Gt][d][pay] at the
+// start of each layer, addressed per token so that a key group's first token t0 (a multiple
+// of Gt) lands on the group's first channel stream; scales [B][H][n_q/Gt][d] likewise.
+void kivi_key_maps(const cg_shape* sh, const cg_params* p, const Sizes& z, RowMap* cm, RowMap* sm) {
+    const int64_t Gt = p->block;
+    cm->base = 0;
+    cm->sL = z.layer_codes;
+    cm->sS = 0;
+    cm->sH = z.key_codes_per_bh;
+    cm->sB = (int64_t)sh->H * cm->sH;
+    cm->sT = (int64_t)sh->d * z.pay / Gt;
+    sm->base = 0;
+    sm->sL = z.layer_scales;
+    sm->sS = 0;
+    sm->sH = z.key_scales_per_bh;
+    sm->sB = (int64_t)sh->H * sm->sH;
+    sm->sT = (int64_t)sh->d / Gt;
+}
+
 // Row map for KIVI values: codes [B][H][n_q][d/blk][pay] after the layer's key part.
 void kivi_value_maps(const cg_shape* sh, const Sizes& z, RowMap* cm, RowMap* sm) {
     const int64_t BH = (int64_t)sh->B * sh->H;
@@ -264,12 +283,21 @@ int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf1
         return CG_OK;
     }
     if (z.nq > 0) {
-        KeyArgs k = key_args(shape, params, z, status);
-        k.x = a.x;
-        k.G = gauges;
-        k.codes = a.codes;
-        k.scales = a.scales;
-        e = launch_key_encode_simt(k, st);
+        RowArgs ka = a;  // keys on tensor cores: s = 0, one block per channel and key group
+        ka.s_lo = 0;
+        ka.s_n = 1;
+        ka.t_count = z.nq;
+        kivi_key_maps(shape, params, z, &ka.cmap, &ka.smap);
+        if (tc_key_encode_eligible(ka)) {
+            e = tc_launch_key_encode(ka, st);
+        } else {
+            KeyArgs k = key_args(shape, params, z, status);
+            k.x = a.x;
+            k.G = gauges;
+            k.codes = a.codes;
+            k.scales = a.scales;
+            e = launch_key_encode_simt(k, st);
+        }
         if (e != cudaSuccess) return cuda_fail(e, "KIVI key encode launch");
         a.s_lo = 1;
         a.s_n = 1;

@@ -190,7 +190,11 @@ __device__ __forceinline__ void patch_code(uint8_t* rowp, int bit, uint32_t q) {
     }
 }
 
-template <int BITS>
+// KEYS = false: block-uniform rows and KIVI value rows (thread = token, block = channels).
+// KEYS = true: KIVI keys (Sec. 4.3, per-channel ranges over a 128-token group): the MMA
+// operands are swapped, D[channel][token] = G x^T, so a thread owns one channel's 128
+// tokens, which form its block and its packed code stream.
+template <int BITS, bool KEYS>
 __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_constant__ CUtensorMap xmap,
                                                                  const EncParams P) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -210,7 +214,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     const int g = a.g, blk = a.blk, npass = kNPass;
     const int gb = g < 16 ? 16 : g;
     const int nbk = kD / blk;
-    const uint32_t bsz = (g == 128) ? 32768u : 16384u;
+    // gauge operand layout: full K = 128 (block-diagonal for g < 128) for keys and g = 128,
+    // else one g-wide K block per group in a 64-column tile
+    const bool fullk = KEYS || g == 128;
+    const uint32_t bsz = fullk ? 32768u : 16384u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
@@ -276,7 +283,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && my_tiles > 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, gb);
+            const uint32_t idesc = idesc_bf16_f32(128, KEYS ? 128 : gb);
+            const int kg = KEYS ? 128 : gb;  // keys: one chain over the full K
             int64_t cur = -1;
             int committed = 0;
             tc::TileIter it;
@@ -301,14 +309,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const uint32_t d_base = tmem + buf * 128;
                 for (int p = 0; p < npass; p++) {
                     const uint32_t b_base = smem_u32(bsplit) + p * bsz;
-                    for (int r = 0; r < 128 / gb; r++) {
-                        for (int ks = 0; ks < gb / 16; ks++) {
-                            const int k0 = r * gb + ks * 16;
+                    for (int r = 0; r < 128 / kg; r++) {
+                        for (int ks = 0; ks < kg / 16; ks++) {
+                            const int k0 = r * kg + ks * 16;
                             const uint32_t a_addr = a_base + (k0 >> 6) * 16384 + (k0 & 63) * 2;
-                            const uint32_t b_addr =
-                                b_base + (g == 128 ? (k0 >> 6) * 16384 : 0) + (r * gb) * 128 + (k0 & 63) * 2;
-                            mma_bf16(d_base + r * gb, sdesc_sw128(a_addr), sdesc_sw128(b_addr), idesc,
-                                     (p > 0 || ks > 0) ? 1u : 0u);
+                            const uint32_t b_addr = b_base + (fullk ? (k0 >> 6) * 16384 : 0) +
+                                                    (KEYS ? 0 : (r * gb) * 128) + (k0 & 63) * 2;
+                            if (KEYS)  // D[channel][token] = G x^T
+                                mma_bf16(d_base, sdesc_sw128(b_addr), sdesc_sw128(a_addr), idesc,
+                                         (p > 0 || ks > 0) ? 1u : 0u);
+                            else  // D[token][channel] = x G^T, one chain per gauge group
+                                mma_bf16(d_base + r * gb, sdesc_sw128(a_addr), sdesc_sw128(b_addr), idesc,
+                                         (p > 0 || ks > 0) ? 1u : 0u);
                         }
                     }
                 }
@@ -327,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         // ------------------------------------------------------------ gauge converter
         const int lg = 31 - __clz(g);
         const float c_order = (float)(1 + lg) * kU * 1.01f;
-        const float c_tc = (float)(npass * (gb / 16) + 2) * kU;
+        const float c_tc = (float)(npass * ((KEYS ? 128 : gb) / 16) + 2) * kU;
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
@@ -397,7 +409,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     }
 #pragma unroll
                     for (int t = 0; t < 3; t++) {
-                        unsigned char* region = bsplit + (npass - 1 - t) * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
+                        unsigned char* region = bsplit + (npass - 1 - t) * bsz + (fullk ? (k >> 6) * 16384 : 0);
                         *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
                             make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
                     }
@@ -406,12 +418,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 #pragma unroll
             for (int q = 0; q < 4; q++)
                 e_row[q] = ((c_order + c_tc) * sqrtf(s_g2[q]) + sqrtf(s_res2[q])) * 1.001f + 1e-30f;
-            // per quantization block: max of e over the rows that bound its values
+            // per quantization block: max of e over the rows that bound its values (keys: a
+            // block is one channel over tokens, bounded by the max over all rows, slot 0)
 #pragma unroll
             for (int bk = 0; bk < 4; bk++) {
-                if (bk < nbk) {
-                    int lo, hi;
-                    bound_range(bk, g, blk, lo, hi);
+                if (KEYS ? bk == 0 : bk < nbk) {
+                    int lo = 0, hi = 128;
+                    if (!KEYS) bound_range(bk, g, blk, lo, hi);
                     float m = 0.0f;
 #pragma unroll
                     for (int q = 0; q < 4; q++) {
@@ -432,7 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         // ------------------------------------------------------------ epilogue warpgroups
         const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup: tiles i = wg (mod 2)
         const int q4 = warp & 3;                      // TMEM lane quadrant of this warp
-        const int row = q4 * 32 + lane;               // tile row = TMEM lane
+        const int row = q4 * 32 + lane;               // TMEM lane: token (rows) or channel (keys)
         const int qw = warp - kEpiWarp0;              // job queue of this warp
         uint32_t* qjob = queue + qw * kQCap * 2;
         const float qmaxf = (float)((1 << BITS) - 1);
@@ -461,14 +474,59 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             }
             tc_fence_after();
             const unsigned char* stg = stages + st * kTileBytes;
-            const bool valid = row < ti.rows_valid;
+            const bool valid = KEYS || row < ti.rows_valid;  // key tiles are whole token groups
             const uint32_t tacc = tmem + ((uint32_t)(q4 * 32) << 16) + buf * 128;
             const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
 
             // ---- 1. ||x||^2 over the bound range of every block (bf16 -> fp32 exact)
             float bs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            if (KEYS) {
+                // a key block is one channel over the tile's 128 tokens: its bound uses the
+                // largest group norm among those tokens; each lane takes 4 token rows, then
+                // the warp reduces (every warp of the group computes it for itself)
+                float gm[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll 1
+                for (int q = 0; q < 4; q++) {
+                    const int tr = lane + 32 * q;
+                    float gs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll 4
-            for (int c8 = 0; c8 < 16; c8++) {
+                    for (int c8 = 0; c8 < 16; c8++) {
+                        const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + tr * 128 +
+                                                                         (((c8 & 7) ^ (tr & 7)) << 4));
+                        float s0 = bf_lo(xv.x) * bf_lo(xv.x);
+                        s0 = fmaf(bf_hi(xv.x), bf_hi(xv.x), s0);
+                        s0 = fmaf(bf_lo(xv.y), bf_lo(xv.y), s0);
+                        s0 = fmaf(bf_hi(xv.y), bf_hi(xv.y), s0);
+                        s0 = fmaf(bf_lo(xv.z), bf_lo(xv.z), s0);
+                        s0 = fmaf(bf_hi(xv.z), bf_hi(xv.z), s0);
+                        s0 = fmaf(bf_lo(xv.w), bf_lo(xv.w), s0);
+                        s0 = fmaf(bf_hi(xv.w), bf_hi(xv.w), s0);
+                        const int r = (c8 * 8) / g;  // g >= 32: at most 4 groups
+#pragma unroll
+                        for (int rr = 0; rr < 4; rr++)
+                            if (rr == r) gs[rr] += s0;
+                    }
+#pragma unroll
+                    for (int rr = 0; rr < 4; rr++) gm[rr] = fmaxf(gm[rr], gs[rr]);
+                    if (!(isfinite(gs[0]) && isfinite(gs[1]) && isfinite(gs[2]) && isfinite(gs[3]))) {
+                        for (int c8 = 0; c8 < 16; c8++) {
+                            const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + tr * 128 +
+                                                                             (((c8 & 7) ^ (tr & 7)) << 4));
+                            const uint32_t wv[4] = {xv.x, xv.y, xv.z, xv.w};
+                            for (int k = 0; k < 4; k++)
+                                if (bf16_nonfinite(wv[k] & 0xffffu) || bf16_nonfinite(wv[k] >> 16))
+                                    flag |= CG_FLAG_NONFINITE_INPUT;
+                        }
+                    }
+                }
+#pragma unroll
+                for (int rr = 0; rr < 4; rr++)
+                    for (int off = 16; off >= 1; off >>= 1)
+                        gm[rr] = fmaxf(gm[rr], __shfl_xor_sync(0xffffffffu, gm[rr], off));
+                bs[0] = pick4(gm, row / g);  // fmaxf keeps a NaN out; non-finite input is flagged above
+            }
+#pragma unroll 4
+            for (int c8 = 0; c8 < (KEYS ? 0 : 16); c8++) {
                 const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
                                                                  (((c8 & 7) ^ (row & 7)) << 4));
                 float s0 = bf_lo(xv.x) * bf_lo(xv.x);
@@ -483,7 +541,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 for (int bk = 0; bk < 4; bk++)
                     if (c8 >= lo8[bk] && c8 < hi8[bk]) bs[bk] += s0;
             }
-            if (valid && !(isfinite(bs[0]) && isfinite(bs[1]) && isfinite(bs[2]) && isfinite(bs[3]))) {
+            if (!KEYS && valid && !(isfinite(bs[0]) && isfinite(bs[1]) && isfinite(bs[2]) && isfinite(bs[3]))) {
                 // a non-finite sum of squares: look for an Inf/NaN input (huge finite values
                 // can also overflow the square)
                 for (int c8 = 0; c8 < 16; c8++) {
@@ -582,7 +640,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                             if (slot >= kQCap) break;
                             const uint32_t col = (uint32_t)(c * 32 + k);
                             const uint32_t tag = col | ((cm & bit) ? 0x100u : 0u) | ((cx & bit) ? 0x200u : 0u);
-                            qjob[2 * slot] = (uint32_t)row | (col << 8);
+                            qjob[2 * slot] = KEYS ? col | ((uint32_t)row << 8) : (uint32_t)row | (col << 8);
                             set4(sl, nm, slot);
                             set4(tg, nm, tag);
                             nm++;
@@ -647,7 +705,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             }
 
             // ---- 6. codes from z~, stored straight from registers; near-boundary values repaired
-            uint8_t* crow = a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
+            // rows: the token's codes; keys: the channel's 128-token stream (16 * BITS bytes)
+            uint8_t* crow = KEYS ? a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0) + (size_t)row * (16 * BITS)
+                                 : a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
             uint32_t am[4] = {0, 0, 0, 0};  // values within mu of a rounding boundary
 #pragma unroll 1
             for (int c = 0; c < 4; c++) {
@@ -731,7 +791,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         const int slot = atomicAdd(&M->qcount[qw], 1);
                         if (slot >= kQCap) break;
                         const int col = c * 32 + k;
-                        qjob[2 * slot] = (uint32_t)row | ((uint32_t)col << 8);
+                        qjob[2 * slot] = KEYS ? (uint32_t)col | ((uint32_t)row << 8) : (uint32_t)row | ((uint32_t)col << 8);
                         set4(sl, nm, slot);
                         set4(cl, nm, col);
                         nm++;
@@ -757,7 +817,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
             // ---- 7. scales; release the stage and the accumulator buffer
             if (valid) {
-                uint32_t* sp = a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
+                uint32_t* sp = KEYS ? a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0) + row
+                                    : a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0 + row);
 #pragma unroll
                 for (int bk = 0; bk < 4; bk++)
                     if (bk < nbk) sp[bk] = s16[bk] | (m16[bk] << 16);
@@ -780,14 +841,34 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     }
 }
 
-template <int BITS>
+template <int BITS, bool KEYS>
 cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
     const size_t smem = EncSmem::total;
-    cudaError_t e = cudaFuncSetAttribute(tc_encode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(tc_encode_kernel<BITS, KEYS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
-    tc_encode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(map, P);
+    tc_encode_kernel<BITS, KEYS><<<(unsigned)grid, kThreads, smem, st>>>(map, P);
     return cudaGetLastError();
+}
+
+template <bool KEYS>
+cudaError_t launch_encode(const RowArgs& a, cudaStream_t st) {
+    EncParams P;
+    P.a = a;
+    P.S = tc::make_sched(a);
+    if (P.S.n_tiles == 0) return cudaSuccess;
+    CUtensorMap map;
+    const uint64_t rows = (uint64_t)a.L * 2 * a.B * a.H * a.T_x;
+    if (!make_tmap_bf16_sw128(&map, a.x, rows, kD, kD * 2, 128)) return cudaErrorInvalidValue;
+    switch (a.bits) {
+        case 2: return launch_encode_bits<2, KEYS>(P, map, st);
+        case 3: return launch_encode_bits<3, KEYS>(P, map, st);
+        case 4: return launch_encode_bits<4, KEYS>(P, map, st);
+        case 6: return launch_encode_bits<6, KEYS>(P, map, st);
+        case 8: return launch_encode_bits<8, KEYS>(P, map, st);
+        default: return cudaErrorInvalidValue;
+    }
 }
 
 }  // namespace
@@ -802,22 +883,20 @@ bool tc_row_encode_eligible(const RowArgs& a) {
     return tmap_encode_fn() != nullptr;
 }
 
-cudaError_t tc_launch_row_encode(const RowArgs& a, cudaStream_t st) {
-    EncParams P;
-    P.a = a;
-    P.S = tc::make_sched(a);
-    if (P.S.n_tiles == 0) return cudaSuccess;
-    CUtensorMap map;
-    const uint64_t rows = (uint64_t)a.L * 2 * a.B * a.H * a.T_x;
-    if (!make_tmap_bf16_sw128(&map, a.x, rows, kD, kD * 2, 128)) return cudaErrorInvalidValue;
-    switch (a.bits) {
-        case 2: return launch_encode_bits<2>(P, map, st);
-        case 3: return launch_encode_bits<3>(P, map, st);
-        case 4: return launch_encode_bits<4>(P, map, st);
-        case 6: return launch_encode_bits<6>(P, map, st);
-        case 8: return launch_encode_bits<8>(P, map, st);
-        default: return cudaErrorInvalidValue;
-    }
+cudaError_t tc_launch_row_encode(const RowArgs& a, cudaStream_t st) { return launch_encode<false>(a, st); }
+
+// KIVI keys as rows of the key tensor: s = 0 only, block = the 128-token key group, t_count
+// = the quantized tokens (whole groups); cmap/smap address a group's first token (the
+// kernel adds the channel's stream). Groups of g >= 32 channels (at most 4 per head).
+bool tc_key_encode_eligible(const RowArgs& a) {
+    if (a.d != kD || a.blk != 128 || a.g < 32) return false;
+    if (a.t_count < 128 || a.t_count % 128) return false;
+    const int64_t rows = (int64_t)a.L * 2 * a.B * a.H * a.T_x;
+    if (rows + 128 >= (int64_t)1 << 31) return false;
+    if ((reinterpret_cast<uintptr_t>(a.x) & 15u) || (reinterpret_cast<uintptr_t>(a.codes) & 15u)) return false;
+    return tmap_encode_fn() != nullptr;
 }
+
+cudaError_t tc_launch_key_encode(const RowArgs& a, cudaStream_t st) { return launch_encode<true>(a, st); }
 
 }  // namespace cg
