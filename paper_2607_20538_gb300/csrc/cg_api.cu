@@ -356,12 +356,21 @@ int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes,
         return CG_OK;
     }
     if (z.nq > 0) {
-        KeyArgs k = key_args(shape, params, z, status);
-        k.out = a.out;
-        k.G = gauges;
-        k.codes = a.codes;
-        k.scales = a.scales;
-        e = launch_key_decode_simt(k, st);
+        RowArgs ka = a;  // keys on tensor cores: s = 0, one 128-token group per tile
+        ka.s_lo = 0;
+        ka.s_n = 1;
+        ka.t_count = z.nq;
+        kivi_key_maps(shape, params, z, &ka.cmap, &ka.smap);
+        if (tc_key_decode_eligible(ka)) {
+            e = tc_launch_key_decode(ka, st);
+        } else {
+            KeyArgs k = key_args(shape, params, z, status);
+            k.out = a.out;
+            k.G = gauges;
+            k.codes = a.codes;
+            k.scales = a.scales;
+            e = launch_key_decode_simt(k, st);
+        }
         if (e != cudaSuccess) return cuda_fail(e, "KIVI key decode launch");
         a.s_lo = 1;
         a.s_n = 1;

@@ -1,0 +1,373 @@
+// cg_tc_keydec.cu -- tensor-core decode of KIVI keys (Sec. 4.3: per-channel key ranges over
+// a token group; Sec. 3: Xhat = G^T Zhat), head dim d = 128, key groups of 128 tokens.
+//
+// A key group stores, per gauge-space channel, a stream of 128 token codes with one scale
+// and zero, so the scale varies along the contraction index of Xhat = G^T Zhat and cannot
+// be applied after the MMA. The unpackers therefore dequantize, zhat = q s + m in fp32, and
+// write zhat as two bf16 terms (hi + lo, 16 significant bits) into a token-major A tile;
+// D[token][i] = sum_j A[token][j] B[i][j] with B = G^T (two bf16 terms) takes three MMA
+// passes (hi·hi, hi·lo, lo·hi; the lo·lo term is below 2^-16 relative).
+//
+// Persistent warp-specialized kernel, one CTA per SM, 10 warps:
+//   warp 0      bulk copy of a group's code streams (128 x 16*bits bytes) and its 128 scales;
+//   warp 1      MMA issuer (24 MMAs per tile, fp32 accumulators, two TMEM buffers);
+//   warps 2..5  one gauge-space channel per thread: unpack, dequantize, split, store the
+//               channel's column of the A tile; at a gauge change they build G^T's split
+//               (full K, block-diagonal for g < 128);
+//   warps 6..9  one token row per thread: accumulator -> bf16 -> global.
+#include <cuda_bf16.h>
+
+#include "cg_sm100.cuh"
+#include "cg_tc.h"
+#include "cg_tc_common.cuh"
+
+namespace cg {
+namespace {
+
+using namespace sm100;
+using tc::kD;
+using tc::kWaitLimitNs;
+
+constexpr int kThreads = 320;
+constexpr int kEpiWarp0 = 6;
+constexpr int kATerm = 128 * kD * 2;  // one bf16 term of a 128 x 128 tile
+constexpr int kAStages = 2;
+constexpr int kSegBufs = 4;
+constexpr int kMma = 3 * 8;           // 3 term pairs x K = 128 in steps of 16
+
+template <int BITS>
+struct KdSmem {
+    static constexpr int cstages_n = BITS >= 4 ? 2 : 4;
+    static constexpr uint32_t cstage_bytes = 128u * 16u * BITS + 512u;  // streams + scales
+    static constexpr uint32_t a_tiles = 0;                              // kAStages x 2 terms
+    static constexpr uint32_t bsplit = a_tiles + kAStages * 2 * kATerm;  // 2 terms x 32 KB
+    static constexpr uint32_t cstages = bsplit + 2 * 32768;
+    static constexpr uint32_t misc = cstages + cstages_n * cstage_bytes;
+    static constexpr uint32_t total = misc + 512;
+    static_assert(cstage_bytes % 16 == 0, "bulk copy sizes are multiples of 16 bytes");
+    static_assert(total + 1024 <= 232448, "shared memory budget");
+};
+
+struct KdMisc {
+    uint64_t cfull[4], cempty[4];
+    uint64_t afull[kAStages], aempty[kAStages];
+    uint64_t accfull[2], accempty[2];
+    uint64_t gready[kSegBufs];
+    uint64_t bfree;
+    uint32_t tmem_slot;
+    int abort_flag;
+};
+static_assert(sizeof(KdMisc) <= 512, "misc block");
+
+struct KdParams {
+    RowArgs a;
+    tc::Sched S;
+};
+
+template <int BITS>
+__global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdParams P) {
+    using SL = KdSmem<BITS>;
+    constexpr int kCStages = SL::cstages_n;
+    constexpr uint32_t kCStageBytes = SL::cstage_bytes;
+    constexpr uint32_t kStreamBytes = 16u * BITS;  // one channel's 128 codes
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const uint32_t base_u32 = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    unsigned char* sm = smem_raw + (base_u32 - smem_u32(smem_raw));
+    KdMisc* M = reinterpret_cast<KdMisc*>(sm + SL::misc);
+    unsigned char* atiles = sm + SL::a_tiles;
+    unsigned char* bsplit = sm + SL::bsplit;
+    unsigned char* cst = sm + SL::cstages;
+
+    const RowArgs& a = P.a;
+    const tc::Sched& S = P.S;
+    const int g = a.g;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+    const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
+    const int64_t t_end = S.n_tiles * (blockIdx.x + 1) / gridDim.x;
+    const int my_tiles = (int)(t_end - t_begin);
+    const int64_t seg0 = my_tiles > 0 ? tc::tile_info(a, S, t_begin).seg : 0;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kCStages; i++) {
+            mbar_init(&M->cfull[i], 1);
+            mbar_init(&M->cempty[i], 4);
+        }
+        for (int i = 0; i < kAStages; i++) {
+            mbar_init(&M->afull[i], 4);
+            mbar_init(&M->aempty[i], 1);
+        }
+        for (int i = 0; i < 2; i++) {
+            mbar_init(&M->accfull[i], 1);
+            mbar_init(&M->accempty[i], 4);
+        }
+        for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 4);
+        mbar_init(&M->bfree, 1);
+        M->abort_flag = 0;
+        fence_barrier_init();
+    }
+    // G^T's split: off-diagonal blocks stay zero for the whole launch
+    for (uint32_t i = threadIdx.x; i < 2u * 32768u / 16u; i += kThreads)
+        reinterpret_cast<uint4*>(bsplit)[i] = make_uint4(0, 0, 0, 0);
+    if (warp == 1) {
+        tmem_alloc(&M->tmem_slot, 256);
+        tmem_relinquish();
+        tc_fence_before();
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = M->tmem_slot;
+    volatile int* abort_flag = &M->abort_flag;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ code/scale producer
+        if (lane == 0 && my_tiles > 0) {
+            int issued = 0;
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+                const int st = i % kCStages;
+                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                const tc::TileInfo ti = it.info(a);
+                unsigned char* dst = cst + st * kCStageBytes;
+                mbar_arrive_expect_tx(&M->cfull[st], 128u * kStreamBytes + 512u);
+                bulk_load(dst, a.codes + a.cmap.at(ti.l, ti.s, ti.b, ti.h, ti.t0), 128u * kStreamBytes, &M->cfull[st]);
+                bulk_load(dst + 128u * kStreamBytes, a.scales + a.smap.at(ti.l, ti.s, ti.b, ti.h, ti.t0), 512u,
+                          &M->cfull[st]);
+                issued = i + 1;
+            }
+            if (*abort_flag) {
+                const int zero = 0;
+                const int from = issued > kCStages ? issued - kCStages : 0;
+                for (int i = from; i < issued; i++)
+                    mbar_wait(&M->cfull[i % kCStages], (i / kCStages) & 1, &zero, kWaitLimitNs);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && my_tiles > 0) {
+            const uint32_t idesc = idesc_bf16_f32(128, 128);
+            const uint64_t bdesc = sdesc_sw128(smem_u32(bsplit));
+            int64_t cur = -1;
+            int committed = 0;
+            tc::TileIter it;
+            it.init(a, S, t_begin);
+            for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+                const tc::TileInfo ti = it.info(a);
+                const int64_t ls = ti.seg - seg0;
+                bool ok = true;
+                if (ti.seg != cur) {
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    cur = ti.seg;
+                }
+                const int ab = i % kAStages, buf = i & 1;
+                ok = ok && mbar_wait(&M->afull[ab], (i / kAStages) & 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                if (!ok) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t adesc = sdesc_sw128(smem_u32(atiles + ab * 2 * kATerm));
+                const uint32_t d_base = tmem + buf * 128;
+#pragma unroll
+                for (int q = 0; q < kMma; q++) {
+                    const int pair = q >> 3, ks = q & 7;  // pairs: (A hi, B hi), (A hi, B lo), (A lo, B hi)
+                    const uint32_t ta = pair == 2 ? 1u : 0u, tb = pair == 1 ? 1u : 0u;
+                    const uint32_t koff = (uint32_t)((ks >> 2) * 16384 + (ks & 3) * 32);  // K = 16 ks
+                    mma_bf16(d_base, adesc + ((ta * kATerm + koff) >> 4), bdesc + ((tb * 32768u + koff) >> 4), idesc,
+                             q > 0 ? 1u : 0u);
+                }
+                mma_commit(&M->accfull[buf]);
+                mma_commit(&M->aempty[ab]);
+                const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
+                if (last_of_seg) mma_commit(&M->bfree);
+                committed = i + 1;
+            }
+            if (*abort_flag && committed > 0) {
+                const int zero = 0;
+                const int i = committed - 1;
+                mbar_wait(&M->accfull[i & 1], (i >> 1) & 1, &zero, kWaitLimitNs);
+            }
+        }
+    } else if (warp < kEpiWarp0) {
+        // ------------------------------------------------------------ unpack + dequantize
+        const int ch = (warp - 2) * 32 + lane;  // gauge-space channel of this thread
+        int64_t cur = -1;
+        int nconv = 0;
+        tc::TileIter it;
+        it.init(a, S, t_begin);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            const tc::TileInfo ti = it.info(a);
+            if (ti.seg != cur) {
+                const int64_t ls = ti.seg - seg0;
+                if (nconv > 0) {
+                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                    if (!__all_sync(0xffffffffu, ok)) {
+                        *abort_flag = 1;
+                        break;
+                    }
+                }
+                // B[n][k] = G_r[k - r g][n - r g] (n, k in group r): thread builds row n = ch
+                const int n = ch, r = n / g, i_in = n - r * g;
+                const float* Gc = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g + (int64_t)r * g * g + i_in;
+                for (int j = 0; j < g; j += 8) {
+                    uint32_t hi[4], lo[4];
+#pragma unroll
+                    for (int e = 0; e < 8; e += 2) {
+                        const float v0 = __ldg(Gc + (int64_t)(j + e) * g);
+                        const float v1 = __ldg(Gc + (int64_t)(j + e + 1) * g);
+                        const __nv_bfloat16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
+                        const __nv_bfloat16 l0 = __float2bfloat16_rn(v0 - __bfloat162float(h0));
+                        const __nv_bfloat16 l1 = __float2bfloat16_rn(v1 - __bfloat162float(h1));
+                        hi[e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+                        lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+                    }
+                    const int k = r * g + j;
+                    const uint32_t off = (k >> 6) * 16384 + sw128_offset(n, k & 63);
+                    *reinterpret_cast<uint4*>(bsplit + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                    *reinterpret_cast<uint4*>(bsplit + 32768 + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
+                cur = ti.seg;
+                nconv++;
+            }
+            const int st = i % kCStages, ab = i % kAStages;
+            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, kWaitLimitNs);
+            ok = ok && mbar_wait(&M->aempty[ab], ((i / kAStages) & 1) ^ 1, abort_flag, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, ok)) {
+                *abort_flag = 1;
+                break;
+            }
+            const unsigned char* stage = cst + st * kCStageBytes;
+            uint32_t w[4 * BITS + 1];
+#pragma unroll
+            for (int q = 0; q < BITS; q++) {
+                const uint4 v = reinterpret_cast<const uint4*>(stage + ch * kStreamBytes)[q];
+                w[4 * q] = v.x;
+                w[4 * q + 1] = v.y;
+                w[4 * q + 2] = v.z;
+                w[4 * q + 3] = v.w;
+            }
+            w[4 * BITS] = 0;
+            const uint32_t sz = reinterpret_cast<const uint32_t*>(stage + 128u * kStreamBytes)[ch];
+            const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
+            const float m = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
+            // column ch of the token-major A tile: token t at row t (128-byte swizzle)
+            unsigned char* ahi = atiles + ab * 2 * kATerm + (ch >> 6) * 16384 + (ch & 7) * 2;
+            unsigned char* alo = ahi + kATerm;
+            const int cu = (ch & 63) >> 3;
+#pragma unroll
+            for (int t = 0; t < 128; t++) {
+                const int p = t * BITS;
+                uint32_t v = w[p >> 5] >> (p & 31);
+                if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
+                const float z = fmaf((float)(v & ((1u << BITS) - 1u)), s, m);
+                const __nv_bfloat16 h = __float2bfloat16_rn(z);
+                const __nv_bfloat16 l = __float2bfloat16_rn(z - __bfloat162float(h));
+                const uint32_t o = t * 128 + ((cu ^ (t & 7)) << 4);
+                *reinterpret_cast<__nv_bfloat16*>(ahi + o) = h;
+                *reinterpret_cast<__nv_bfloat16*>(alo + o) = l;
+            }
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(&M->afull[ab]);
+                mbar_arrive(&M->cempty[st]);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int q4 = warp & 3;
+        const int row = q4 * 32 + lane;  // token of the group
+        tc::TileIter it;
+        it.init(a, S, t_begin);
+        for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
+            const tc::TileInfo ti = it.info(a);
+            const int buf = i & 1;
+            const bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+            if (!__all_sync(0xffffffffu, ok)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t tacc = tmem + ((uint32_t)(q4 * 32) << 16) + buf * 128;
+            uint4* orow = reinterpret_cast<uint4*>(a.out + (tc::dense_row(a, ti) + row) * kD);
+#pragma unroll 1
+            for (int c = 0; c < 4; c++) {
+                uint32_t v[32];
+                tmem_ld32(tacc + c * 32, v);
+                tmem_wait_ld();
+                if (c == 3) {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&M->accempty[buf]);
+                }
+                uint32_t o[16];
+#pragma unroll
+                for (int e = 0; e < 16; e++) {
+                    const __nv_bfloat162 b2 = __floats2bfloat162_rn(__uint_as_float(v[2 * e]), __uint_as_float(v[2 * e + 1]));
+                    o[e] = *reinterpret_cast<const uint32_t*>(&b2);
+                }
+#pragma unroll
+                for (int q = 0; q < 4; q++) orow[c * 4 + q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+            }
+        }
+    }
+    __syncthreads();
+    if (*abort_flag && threadIdx.x == 0) raise_flag(a.status, CG_FLAG_PIPE_TIMEOUT);
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(tmem, 256);
+    }
+}
+
+template <int BITS>
+cudaError_t launch_kd(const KdParams& P, cudaStream_t st) {
+    const size_t smem = KdSmem<BITS>::total + 1024;
+    cudaError_t e =
+        cudaFuncSetAttribute(tc_key_decode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
+    tc_key_decode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(P);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+// KIVI keys as rows of the key tensor (s = 0, t_count = the quantized tokens, whole
+// 128-token groups); cmap/smap address a group's first channel stream and scale.
+bool tc_key_decode_eligible(const RowArgs& a) {
+    if (a.d != kD || a.blk != 128) return false;
+    if (a.t_count < 128 || a.t_count % 128) return false;
+    const int64_t rows = (int64_t)a.L * 2 * a.B * a.H * a.T_x;
+    if (rows + 128 >= (int64_t)1 << 31) return false;
+    if ((reinterpret_cast<uintptr_t>(a.codes) & 15u) || (reinterpret_cast<uintptr_t>(a.scales) & 15u) ||
+        (reinterpret_cast<uintptr_t>(a.out) & 15u))
+        return false;
+    return true;
+}
+
+cudaError_t tc_launch_key_decode(const RowArgs& a, cudaStream_t st) {
+    KdParams P;
+    P.a = a;
+    P.S = tc::make_sched(a);
+    if (P.S.n_tiles == 0) return cudaSuccess;
+    switch (a.bits) {
+        case 2: return launch_kd<2>(P, st);
+        case 3: return launch_kd<3>(P, st);
+        case 4: return launch_kd<4>(P, st);
+        case 6: return launch_kd<6>(P, st);
+        case 8: return launch_kd<8>(P, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace cg
