@@ -64,7 +64,7 @@ struct EncSmem {
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
     static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 8 warps x kQCap x 8 B
     static constexpr uint32_t misc = queue + 8 * kQCap * 8;
-    static constexpr uint32_t total = misc + 320;  // base is 1024-aligned (checked in-kernel)
+    static constexpr uint32_t total = misc + 384;  // base is 1024-aligned (checked in-kernel)
 };
 
 struct Misc {
@@ -76,9 +76,10 @@ struct Misc {
     int abort_flag;
     int qcount[8];
     float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
+    float gmaxb[kSegBufs][4];  // and max_i ||G_i||
 };
 
-static_assert(sizeof(Misc) <= 320, "Misc outgrew its shared-memory slot");
+static_assert(sizeof(Misc) <= 384, "Misc outgrew its shared-memory slot");
 static_assert(EncSmem::total <= 232448, "encode kernel exceeds 227 KB of shared memory");
 
 struct EncParams {
@@ -431,8 +432,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         const int n = lane + 32 * q;
                         if (n >= lo && n < hi) m = fmaxf(m, e_row[q]);
                     }
-                    for (int off = 16; off >= 1; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-                    if (lane == 0) M->emaxb[ls & 3][bk] = m;
+                    float gm = 0.0f;  // max_i ||G_i|| over the same rows: bounds |z~| / ||x||
+#pragma unroll
+                    for (int q = 0; q < 4; q++) {
+                        const int n = lane + 32 * q;
+                        if (n >= lo && n < hi) gm = fmaxf(gm, sqrtf(s_g2[q]));
+                    }
+                    for (int off = 16; off >= 1; off >>= 1) {
+                        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+                        gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, off));
+                    }
+                    if (lane == 0) {
+                        M->emaxb[ls & 3][bk] = m;
+                        M->gmaxb[ls & 3][bk] = gm;
+                    }
                 }
             }
             fence_proxy_async_smem();
@@ -553,9 +566,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
 
-            // ---- 2. approximate block ranges from the accumulator
+            // ---- 2. approximate block ranges from the accumulator, and per 32-column chunk the
+            // values within 2 Ep of the chunk's own min / max, Ep >= E (item 3) being known
+            // before the ranges are: any candidate extreme of a block is among them
             float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
             float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+            float clo[4], chi[4];           // chunk min / max
+            uint32_t pm[4], px[4];          // chunk candidate masks (bit k = column 32c + k)
 #pragma unroll 1
             for (int c = 0; c < 4; c++) {
                 uint32_t v[32];
@@ -572,6 +589,22 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const int bk = (c * 32) / blk;
                 set4(mn, bk, fminf(pick4(mn, bk), lo));
                 set4(mx, bk, fmaxf(pick4(mx, bk), hi));
+                // |z~| <= ||G_i|| ||x|| + E, so Ep bounds the E of item 3 from above
+                const float xn = sqrtf(pick4(bs, bk)) * 1.0001f;
+                const float ep = xn * M->emaxb[ls & 3][bk] + 2.0f * xn * M->gmaxb[ls & 3][bk] * 2.41e-7f;
+                const float tl = __fadd_rn(lo, 2.0f * ep), th = __fsub_rn(hi, 2.0f * ep);
+                // sign bits of (threshold - z) and (z - threshold), shifted in from column 31 down
+                uint32_t a0 = 0, a1 = 0;
+#pragma unroll
+                for (int k = 31; k >= 0; k--) {
+                    const float z = __uint_as_float(v[k]);
+                    a0 = __funnelshift_l(__float_as_uint(__fsub_rn(tl, z)), a0, 1);
+                    a1 = __funnelshift_l(__float_as_uint(__fsub_rn(z, th)), a1, 1);
+                }
+                set4(clo, c, lo);
+                set4(chi, c, hi);
+                set4(pm, c, ~a0);  // z <= tl
+                set4(px, c, ~a1);  // z >= th
             }
 
             // ---- 3. error bound per block; scale/zero from the intervals when they agree
@@ -599,27 +632,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
             // ---- 4. exact extremes of ambiguous blocks (warp-cooperative rounds)
             if (__any_sync(0xffffffffu, amb != 0)) {
-                // candidate masks per 32-column chunk: values within 2E of the block's min / max
-                uint32_t pm[4] = {0, 0, 0, 0}, px[4] = {0, 0, 0, 0};
+                // candidates: a chunk's values near its own min (max) are candidates of the
+                // block min (max) when the chunk min lies within 2E of the block min
 #pragma unroll 1
                 for (int c = 0; c < 4; c++) {
                     const int bk = (c * 32) / blk;
                     const int need = (amb >> (2 * bk)) & 3;
-                    if (!__any_sync(0xffffffffu, need != 0)) continue;
-                    uint32_t v[32];
-                    tmem_ld32(tacc + c * 32, v);
-                    tmem_wait_ld();
                     const float e2 = 2.0f * pick4(E, bk);
-                    const float thr_lo = __fadd_rn(pick4(mn, bk), e2), thr_hi = __fsub_rn(pick4(mx, bk), e2);
-                    uint32_t a0 = 0, a1 = 0;
-#pragma unroll
-                    for (int k = 0; k < 32; k++) {
-                        const float z = __uint_as_float(v[k]);
-                        if (z <= thr_lo) a0 |= 1u << k;
-                        if (z >= thr_hi) a1 |= 1u << k;
-                    }
-                    set4(pm, c, need ? a0 : 0u);
-                    set4(px, c, (need & 1) ? a1 : 0u);
+                    const bool nl = need && pick4(clo, c) <= __fadd_rn(pick4(mn, bk), e2);
+                    const bool nh = (need & 1) && pick4(chi, c) >= __fsub_rn(pick4(mx, bk), e2);
+                    set4(pm, c, nl ? pick4(pm, c) : 0u);
+                    set4(px, c, nh ? pick4(px, c) : 0u);
                 }
                 float ex_mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
                 float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
