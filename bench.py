@@ -120,10 +120,11 @@ class Clocks:
                 "samples": len(sm)}
 
 
-def _kernel_traffic(kind: str):
-    """ncu DRAM bytes per launch recorded in profiles/traffic.json, or None when the kernel
+def _kernel_traffic(kind: str, workload: str):
+    """ncu DRAM bytes (read + write) per launch of the kernel on this workload, recorded in
+    profiles/dram_traffic_<workload>.json, or None when there is no record or the kernel
     source changed since the counters were taken."""
-    p = os.path.join(ROOT, "profiles", "traffic.json")
+    p = os.path.join(ROOT, "profiles", f"dram_traffic_{workload}.json")
     try:
         rec = json.load(open(p))[kind]
     except Exception:
@@ -312,7 +313,8 @@ def run_cuda(args):
             "encode_ms": round(enc_avg, 5), "decode_ms": round(dec_avg, 5),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 2), "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": _kernel_traffic(dom), "alg_bytes_per_launch": dom_alg,
+                         "traffic": None if args.layers else _kernel_traffic(dom, w.name),
+                         "alg_bytes_per_launch": dom_alg,
                          "enc_frac": round(enc_alg / (enc_avg * 1e-3) / 1e9 / peak, 4),
                          "dec_frac": round(dec_alg / (dec_avg * 1e-3) / 1e9 / peak, 4)},
             "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": n_bf16,
