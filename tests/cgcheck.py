@@ -1,6 +1,6 @@
 """Parity helpers: run the CUDA path through the C ABI and compare with the CPU oracle.
 
-Tolerances (the benchmark spec of the hot path, with this build's readings):
+Tolerances (the accepted error of the method's outputs, with the library's readings):
   - packed byte counts and layout: exact;
   - codes: bit-exact, except elements the oracle flags (pre-rounding value within 1e-4
     steps of a rounding boundary), which may differ by +-1; at most 1e-4 of all elements;
