@@ -23,6 +23,7 @@ def nvcc() -> str:
 
 def _flags(extra=()):
     return [*ARCH, "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
+            "-Xcompiler", "-fvisibility=hidden",
             "--expt-relaxed-constexpr", *extra]
 
 

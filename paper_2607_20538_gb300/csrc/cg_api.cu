@@ -10,6 +10,9 @@
 #include "cg_launch.h"
 #include "cg_tc.h"
 
+// The library is built with hidden symbol visibility; only the C ABI is exported.
+#define CG_EXPORT __attribute__((visibility("default")))
+
 namespace cg {
 
 __device__ int32_t g_status_word = 0;
@@ -234,9 +237,9 @@ using namespace cg;
 
 extern "C" {
 
-const char* cg_last_error(void) { return t_err.c_str(); }
+CG_EXPORT const char* cg_last_error(void) { return t_err.c_str(); }
 
-int cg_packed_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes, size_t* scales_bytes,
+CG_EXPORT int cg_packed_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes, size_t* scales_bytes,
                     size_t* residual_bytes) {
     t_err.clear();
     Sizes z;
@@ -248,7 +251,7 @@ int cg_packed_bytes(const cg_shape* shape, const cg_params* params, size_t* code
     return CG_OK;
 }
 
-int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf16, const float* gauges,
+CG_EXPORT int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf16, const float* gauges,
               void* out_codes, void* out_scales, void* out_residual, void* stream) {
     t_err.clear();
     Sizes z;
@@ -321,7 +324,7 @@ int cg_encode(const cg_shape* shape, const cg_params* params, const void* kv_bf1
     return CG_OK;
 }
 
-int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes, const void* scales,
+CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes, const void* scales,
               const void* residual, const float* gauges, void* out_kv_bf16, void* stream) {
     t_err.clear();
     Sizes z;
@@ -394,7 +397,7 @@ int cg_decode(const cg_shape* shape, const cg_params* params, const void* codes,
     return CG_OK;
 }
 
-int cg_get_status(void* stream, int32_t* device_flags) {
+CG_EXPORT int cg_get_status(void* stream, int32_t* device_flags) {
     t_err.clear();
     if (!device_flags) return fail(CG_EINVAL, "null device_flags");
     int32_t* status = nullptr;
