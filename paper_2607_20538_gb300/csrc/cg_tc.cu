@@ -648,42 +648,54 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                 bool pend = (pm[0] | pm[1] | pm[2] | pm[3] | px[0] | px[1] | px[2] | px[3]) != 0;
                 while (__any_sync(0xffffffffu, pend)) {
-                    if (lane == 0) M->qcount[qw] = 0;
-                    __syncwarp();
-                    int sl[kMine] = {0, 0, 0, 0};
-                    uint32_t tg[kMine] = {0, 0, 0, 0};
-                    int nm = 0;
+                    // every lane's candidates take consecutive slots (warp prefix sum of the
+                    // counts); one cooperative round serves up to kQCap of them
+                    const int cnt = __popc(pm[0] | px[0]) + __popc(pm[1] | px[1]) + __popc(pm[2] | px[2]) +
+                                    __popc(pm[3] | px[3]);
+                    int inc = cnt;
+#pragma unroll
+                    for (int off = 1; off < 32; off <<= 1) {
+                        const int t = __shfl_up_sync(0xffffffffu, inc, off);
+                        if (lane >= off) inc += t;
+                    }
+                    const int base = inc - cnt;
+                    const int total = __shfl_sync(0xffffffffu, inc, 31);
+                    int slot = base;
 #pragma unroll 1
-                    for (int c = 0; c < 4; c++) {
-                        uint32_t cm = pick4(pm, c), cx = pick4(px, c);
-                        while (nm < kMine && (cm | cx)) {
-                            const int k = __ffs(cm | cx) - 1;
-                            const uint32_t bit = 1u << k;
-                            const int slot = atomicAdd(&M->qcount[qw], 1);
-                            if (slot >= kQCap) break;
-                            const uint32_t col = (uint32_t)(c * 32 + k);
-                            const uint32_t tag = col | ((cm & bit) ? 0x100u : 0u) | ((cx & bit) ? 0x200u : 0u);
+                    for (int c = 0; c < 4 && slot < kQCap; c++) {
+                        uint32_t m = pick4(pm, c) | pick4(px, c);
+                        while (m && slot < kQCap) {
+                            const uint32_t col = (uint32_t)(c * 32 + __ffs(m) - 1);
                             qjob[2 * slot] = KEYS ? col | ((uint32_t)row << 8) : (uint32_t)row | (col << 8);
-                            set4(sl, nm, slot);
-                            set4(tg, nm, tag);
-                            nm++;
-                            cm &= ~bit;
-                            cx &= ~bit;
+                            m &= m - 1;
+                            slot++;
                         }
-                        set4(pm, c, cm);
-                        set4(px, c, cx);
                     }
                     __syncwarp();
-                    const int nq = min(M->qcount[qw], kQCap);
-                    run_jobs(qjob, nq, stg, Gf, g, lane);
+                    run_jobs(qjob, min(total, kQCap), stg, Gf, g, lane);
                     __syncwarp();
+                    // the same candidates in the same order: fold the exact values in
+                    slot = base;
 #pragma unroll 1
-                    for (int m = 0; m < nm; m++) {
-                        const uint32_t tgm = pick4(tg, m);
-                        const float ze = __uint_as_float(qjob[2 * pick4(sl, m) + 1]);
-                        const int bk = (int)(tgm & 0xffu) / blk;
-                        if (tgm & 0x100u) set4(ex_mn, bk, fminf(pick4(ex_mn, bk), ze));
-                        if (tgm & 0x200u) set4(ex_mx, bk, fmaxf(pick4(ex_mx, bk), ze));
+                    for (int c = 0; c < 4 && slot < kQCap; c++) {
+                        uint32_t cm = pick4(pm, c), cx = pick4(px, c);
+                        uint32_t m = cm | cx;
+                        const int bk = (c * 32) / blk;
+                        float emn = pick4(ex_mn, bk), emx = pick4(ex_mx, bk);
+                        while (m && slot < kQCap) {
+                            const uint32_t bit = m & (0u - m);
+                            const float ze = __uint_as_float(qjob[2 * slot + 1]);
+                            if (cm & bit) emn = fminf(emn, ze);
+                            if (cx & bit) emx = fmaxf(emx, ze);
+                            cm &= ~bit;
+                            cx &= ~bit;
+                            m &= m - 1;
+                            slot++;
+                        }
+                        set4(ex_mn, bk, emn);
+                        set4(ex_mx, bk, emx);
+                        set4(pm, c, cm);
+                        set4(px, c, cx);
                     }
                     __syncwarp();
                     pend = (pm[0] | pm[1] | pm[2] | pm[3] | px[0] | px[1] | px[2] | px[3]) != 0;
