@@ -52,7 +52,6 @@ constexpr int kTileBytes = 128 * kD * 2;
 constexpr int kThreads = 352;
 constexpr int kEpiWarp0 = 3;
 constexpr int kQCap = 32;             // repair jobs per warp and round
-constexpr int kMine = 4;              // jobs one thread queues per round
 constexpr int kAcc = 4;               // accumulator buffers in tensor memory
 constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
@@ -74,7 +73,6 @@ struct Misc {
     uint64_t bfree;
     uint32_t tmem_slot;
     int abort_flag;
-    int qcount[8];
     float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
     float gmaxb[kSegBufs][4];  // and max_i ||G_i||
 };
@@ -814,37 +812,43 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             }
             bool pend = (am[0] | am[1] | am[2] | am[3]) != 0;
             while (__any_sync(0xffffffffu, pend)) {
-                if (lane == 0) M->qcount[qw] = 0;
-                __syncwarp();
-                int sl[kMine] = {0, 0, 0, 0}, cl[kMine] = {0, 0, 0, 0};
-                int nm = 0;
+                const int cnt = __popc(am[0]) + __popc(am[1]) + __popc(am[2]) + __popc(am[3]);
+                int inc = cnt;
+#pragma unroll
+                for (int off = 1; off < 32; off <<= 1) {
+                    const int t = __shfl_up_sync(0xffffffffu, inc, off);
+                    if (lane >= off) inc += t;
+                }
+                const int base = inc - cnt;
+                const int total = __shfl_sync(0xffffffffu, inc, 31);
+                int slot = base;
 #pragma unroll 1
-                for (int c = 0; c < 4; c++) {
-                    uint32_t ca = pick4(am, c);
-                    while (nm < kMine && ca) {
-                        const int k = __ffs(ca) - 1;
-                        const int slot = atomicAdd(&M->qcount[qw], 1);
-                        if (slot >= kQCap) break;
-                        const int col = c * 32 + k;
-                        qjob[2 * slot] = KEYS ? (uint32_t)col | ((uint32_t)row << 8) : (uint32_t)row | ((uint32_t)col << 8);
-                        set4(sl, nm, slot);
-                        set4(cl, nm, col);
-                        nm++;
-                        ca &= ca - 1;
+                for (int c = 0; c < 4 && slot < kQCap; c++) {
+                    uint32_t m = pick4(am, c);
+                    while (m && slot < kQCap) {
+                        const uint32_t col = (uint32_t)(c * 32 + __ffs(m) - 1);
+                        qjob[2 * slot] = KEYS ? col | ((uint32_t)row << 8) : (uint32_t)row | (col << 8);
+                        m &= m - 1;
+                        slot++;
                     }
-                    set4(am, c, ca);
                 }
                 __syncwarp();
-                const int nq = min(M->qcount[qw], kQCap);
-                run_jobs(qjob, nq, stg, Gf, g, lane);
+                run_jobs(qjob, min(total, kQCap), stg, Gf, g, lane);
                 __syncwarp();
+                slot = base;
 #pragma unroll 1
-                for (int m = 0; m < nm; m++) {
-                    const int col = pick4(cl, m);
-                    const float ze = __uint_as_float(qjob[2 * pick4(sl, m) + 1]);
-                    const int bk = col / blk;
-                    const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
-                    patch_code<BITS>(crow, col * BITS, q);
+                for (int c = 0; c < 4 && slot < kQCap; c++) {
+                    uint32_t m = pick4(am, c);
+                    while (m && slot < kQCap) {
+                        const int col = c * 32 + __ffs(m) - 1;
+                        const float ze = __uint_as_float(qjob[2 * slot + 1]);
+                        const int bk = col / blk;
+                        const uint32_t q = quant_code(ze, h2f_bits(pick4(s16, bk)), h2f_bits(pick4(m16, bk)), qmax);
+                        patch_code<BITS>(crow, col * BITS, q);
+                        m &= m - 1;
+                        slot++;
+                    }
+                    set4(am, c, m);
                 }
                 __syncwarp();
                 pend = (am[0] | am[1] | am[2] | am[3]) != 0;
