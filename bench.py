@@ -142,31 +142,35 @@ def _kernel_traffic(kind: str, workload: str):
     return rec["bytes_per_launch"] if h == rec["source_sha"] else None
 
 
-def cpu_sample(w, G, seconds=12.0, nthreads=None):
-    """Time the oracle (as it stands) on whole (l, s, b, h) units of the workload."""
+def cpu_sample(w, G, seconds=12.0, nthreads=None, start=0):
+    """Time the oracle (as it stands) on whole (layer, sequence) slices of the workload: the K and
+    V units of every head of one (l, b), one slice after the other from slice `start`, until
+    `seconds` of oracle time have accumulated (at least one slice)."""
     import numpy as np
 
     import oracle
     from paper_2607_20538_gb300 import synth
     nthreads = nthreads or os.cpu_count() or 1
-    done_bytes, t_total, layers = 0, 0.0, 0
-    for l in range(w.L):
-        sub = w.replace(L=1)
-        x = np.stack([np.stack([np.stack([np.stack([synth.kv_unit(w, l, s, b, h) for h in range(w.H)])
-                                          for b in range(w.B)]) for s in range(2)])])
+    sub = w.replace(L=1, B=1, T_cap=0)
+    done_bytes, t_total, n = 0, 0.0, 0
+    n_slices = w.L * w.B
+    while n < n_slices:
+        l, b = divmod((start + n) % n_slices, w.B)
+        x = np.stack([np.stack([np.stack([synth.kv_unit(w, l, s, b, h) for h in range(w.H)])
+                                for s in range(2)])])[:, :, None]
         Gl = np.ascontiguousarray(G[l:l + 1])
         t0 = time.perf_counter()
         r = oracle.encode(sub.shape, sub.params, x, Gl, nthreads=nthreads)
         oracle.decode(sub.shape, sub.params, r["codes"], r["scales"], r["residual"], Gl, nthreads=nthreads)
         t_total += time.perf_counter() - t0
         done_bytes += 2 * x.nbytes
-        layers += 1
+        n += 1
         if t_total >= seconds:
             break
     return {"value": done_bytes / t_total / 1e9, "unit": "GB/s", "cores": nthreads, "kind": "oracle",
-            "sample": f"encode+decode of {layers} of {w.L} layers of the {w.name} cache "
-                      f"({layers * 2 * w.B * w.H} (l,s,b,h) units, {done_bytes // 2} bf16 bytes), "
-                      f"{t_total:.1f} s on {nthreads} threads"}
+            "sample": f"encode+decode of {n} of {n_slices} (layer, sequence) slices of the {w.name} cache "
+                      f"({n * 2 * w.H} (l,s,b,h) units, {done_bytes // 2} bf16 bytes), "
+                      f"{t_total:.2f} s on {nthreads} threads"}
 
 
 def run_reference(args):
@@ -179,12 +183,13 @@ def run_reference(args):
         w = w.replace(L=min(args.layers, w.L))
     G = synth.gauges(w)
     cores = os.cpu_count() or 1
-    for _ in range(args.warmup):
-        cpu_sample(w.replace(L=1), G, seconds=0.0, nthreads=cores)
+    for i in range(args.warmup):
+        cpu_sample(w, G, seconds=0.0, nthreads=cores, start=i)
     vals = []
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        vals.append(cpu_sample(w, G, seconds=1.0, nthreads=cores))
+    for i in range(args.steps):
+        # one step: a bounded sample (one or more (layer, sequence) slices, ~0.25 s)
+        vals.append(cpu_sample(w, G, seconds=0.25, nthreads=cores, start=args.warmup + i))
     el = time.perf_counter() - t0
     v = statistics.median(x["value"] for x in vals)
     line = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s", "n_gpus": args.gpus,
@@ -197,8 +202,116 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def run_cuda(args):
+class _Problem:
+    """What one step runs and how its bytes count (set up by _setup_cache / _setup_rolling)."""
+
+
+def _setup_cache(w, dev, ws, stream):
+    """Whole-cache step: encode the workload's cache, then decode it."""
     import numpy as np
+    import torch
+
+    import paper_2607_20538_gb300 as cg
+    from paper_2607_20538_gb300 import synth
+    P = _Problem()
+    shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
+    nc, ns, nr = cg.packed_bytes(shape, params)
+    x = synth.kv_cache(w, threads=max(4, (os.cpu_count() or 8) // max(ws, 1)))
+    P.G = synth.gauges(w)
+    dx = torch.from_numpy(x.reshape(-1).view(np.int16)).to(dev)
+    dG = torch.from_numpy(P.G.reshape(-1)).to(dev)
+    codes, scales, resid = cg.alloc_outputs(shape, params, device=dev)
+    out = torch.empty_like(dx)
+    n = x.nbytes
+    P.enc_bytes = P.dec_bytes = n
+    P.enc_alg = P.dec_alg = n + nc + ns + nr + P.G.nbytes
+    P.launches = 2 if w.backend != 1 else 2 * 3
+    P.config = {}
+
+    def encode():
+        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+
+    def decode():
+        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
+
+    P.encode, P.decode = encode, decode
+    hx = torch.from_numpy(x.reshape(-1).view(np.int16)).pin_memory()
+    hout = torch.empty_like(hx).pin_memory()
+
+    def e2e_step():
+        dx.copy_(hx, non_blocking=True)
+        encode()
+        decode()
+        hout.copy_(out, non_blocking=True)
+
+    P.e2e_step, P.h2d, P.d2h = e2e_step, n, n
+    P.e2e_bytes = 2 * n
+    return P
+
+
+def _setup_rolling(w, dev, ws, stream):
+    """Rolling decode step over a history of T_cap tokens per sequence: encode one new token per
+    sequence into position T_cap - 1, then decode the whole history. The history is encoded once
+    before timing (layer by layer; every layer holds one draw of layer 0's tokens, see synth)."""
+    import numpy as np
+    import torch
+
+    import paper_2607_20538_gb300 as cg
+    from paper_2607_20538_gb300 import synth
+    P = _Problem()
+    Tc = w.T_cap
+    params = cg.Params(**w.params)
+    full = cg.Shape(L=w.L, B=w.B, H=w.H, T=Tc, d=w.d, t0=0, T_cap=Tc)
+    app = cg.Shape(L=w.L, B=w.B, H=w.H, T=1, d=w.d, t0=Tc - 1, T_cap=Tc)
+    lay = cg.Shape(L=1, B=w.B, H=w.H, T=Tc - 1, d=w.d, t0=0, T_cap=Tc)
+    nc, ns, _ = cg.packed_bytes(full, params)
+    nc1, ns1, _ = cg.packed_bytes(lay, params)
+    P.G = synth.gauges(w)
+    dG = torch.from_numpy(P.G.reshape(-1)).to(dev)
+    codes, scales, _ = cg.alloc_outputs(full, params, device=dev)
+    threads = max(4, (os.cpu_count() or 8) // max(ws, 1))
+    dh = torch.from_numpy(synth.rolling_history_layer(w, threads=threads).reshape(-1).view(np.int16)).to(dev)
+    per_g = dG.numel() // w.L
+    for l in range(w.L):
+        cg.encode(lay, params, dh, dG[l * per_g:(l + 1) * per_g], codes[l * nc1:(l + 1) * nc1],
+                  scales[l * ns1 // 4:(l + 1) * ns1 // 4], None, stream=stream)
+    del dh
+    xnew = synth.rolling_new_token(w, threads=threads)
+    dnew = torch.from_numpy(xnew.reshape(-1).view(np.int16)).to(dev)
+    n_out = w.L * 2 * w.B * w.H * Tc * w.d
+    out = torch.empty(n_out, dtype=torch.int16, device=dev)
+    P.enc_bytes, P.dec_bytes = xnew.nbytes, 2 * n_out
+    tok_codes = w.L * 2 * w.B * w.H * (w.d * w.bits // 8)
+    tok_scales = w.L * 2 * w.B * w.H * (w.d // w.block) * 4
+    P.enc_alg = xnew.nbytes + tok_codes + tok_scales + P.G.nbytes
+    P.dec_alg = nc + ns + P.G.nbytes + 2 * n_out
+    P.launches = 2
+    P.config = {"T_cap": Tc, "step": "append 1 token per sequence at T_cap - 1, decode all T_cap tokens"}
+
+    def encode():
+        cg.encode(app, params, dnew, dG, codes, scales, None, stream=stream)
+
+    def decode():
+        cg.decode(full, params, codes, scales, None, dG, out, stream=stream)
+
+    P.encode, P.decode = encode, decode
+    hnew = torch.from_numpy(xnew.reshape(-1).view(np.int16)).pin_memory()
+    last = out.view(w.L * 2 * w.B * w.H, Tc, w.d)[:, Tc - 1, :]
+    hlast = torch.empty(last.shape, dtype=torch.int16).pin_memory()
+
+    def e2e_step():
+        # the new tokens in, the step, and the decoded newest token of every sequence out
+        dnew.copy_(hnew, non_blocking=True)
+        encode()
+        decode()
+        hlast.copy_(last, non_blocking=True)
+
+    P.e2e_step, P.h2d, P.d2h = e2e_step, hnew.numel() * 2, hlast.numel() * 2
+    P.e2e_bytes = P.enc_bytes + P.dec_bytes
+    return P
+
+
+def run_cuda(args):
     import torch
 
     import paper_2607_20538_gb300 as cg
@@ -215,25 +328,16 @@ def run_cuda(args):
     w = synth.WORKLOADS[args.workload]
     if args.layers:
         w = w.replace(L=min(args.layers, w.L))
-    shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
-    nc, ns, nr = cg.packed_bytes(shape, params)
-    x = synth.kv_cache(w, threads=max(4, (os.cpu_count() or 8) // max(ws, 1)))
-    G = synth.gauges(w)
-    dx = torch.from_numpy(x.reshape(-1).view(np.int16)).to(dev)
-    dG = torch.from_numpy(G.reshape(-1)).to(dev)
-    codes, scales, resid = cg.alloc_outputs(shape, params, device=dev)
-    out = torch.empty_like(dx)
     stream = torch.cuda.current_stream()
-    n_bf16 = x.nbytes
-    g_bytes = G.nbytes
+    P = (_setup_rolling if w.T_cap else _setup_cache)(w, dev, ws, stream)
 
     def step(ev=None):
         if ev is not None:
             ev[0].record(stream)
-        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+        P.encode()
         if ev is not None:
             ev[1].record(stream)
-        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
+        P.decode()
         if ev is not None:
             ev[2].record(stream)
 
@@ -264,71 +368,61 @@ def run_cuda(args):
     dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
     total_ms = rank_reduce(total_ms, "max", dev)
     ms_step = total_ms / args.steps
-    value = job_throughput(2 * n_bf16, ws, ms_step)
+    value = job_throughput(P.enc_bytes + P.dec_bytes, ws, ms_step)
     enc_avg, dec_avg = statistics.mean(enc_ms), statistics.mean(dec_ms)
-    enc_alg = n_bf16 + nc + ns + nr + g_bytes
-    dec_alg = nc + ns + nr + g_bytes + n_bf16
     peak, peak_kind = _peaks()
     if dec_avg >= enc_avg:
-        dom, dom_ms, dom_alg = "decode", dec_avg, dec_alg
+        dom, dom_ms, dom_alg = "decode", dec_avg, P.dec_alg
     else:
-        dom, dom_ms, dom_alg = "encode", enc_avg, enc_alg
+        dom, dom_ms, dom_alg = "encode", enc_avg, P.enc_alg
     achieved = dom_alg / (dom_ms * 1e-3) / 1e9
 
     # end to end through the C ABI with host buffers
-    hx = torch.from_numpy(x.reshape(-1).view(np.int16)).pin_memory()
-    hout = torch.empty_like(hx).pin_memory()
     e2e_steps = max(3, min(args.steps, 20))
-
-    def e2e_step():
-        dx.copy_(hx, non_blocking=True)
-        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
-        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
-        hout.copy_(out, non_blocking=True)
-
     for _ in range(2):
-        e2e_step()
+        P.e2e_step()
     torch.cuda.synchronize()
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(e2e_steps):
-        e2e_step()
+        P.e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = rank_reduce(e0.elapsed_time(e1) / e2e_steps, "max", dev)
-    e2e_val = job_throughput(2 * n_bf16, ws, e2e_ms)
+    e2e_val = job_throughput(P.e2e_bytes, ws, e2e_ms)
     flags = cg.get_status()
     if flags:
         raise RuntimeError(f"device status flags {flags} after the timed region")
 
     if rank == 0:
-        launches_per_step = 2 if w.backend != 1 else 2 * (1 + 1 + 1)
+        config = {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
+                  "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
+                  "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
+                  "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
+                  "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"}
+        config.update(P.config)
         line = {
             "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms_step, 5), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
-                       "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
-                       "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
-                       "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
-                       "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"},
-            "encode_gbs": round(n_bf16 / (enc_avg * 1e-3) / 1e9, 2),
-            "decode_gbs": round(n_bf16 / (dec_avg * 1e-3) / 1e9, 2),
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic", "config": config,
+            "encode_gbs": round(P.enc_bytes / (enc_avg * 1e-3) / 1e9, 2),
+            "decode_gbs": round(P.dec_bytes / (dec_avg * 1e-3) / 1e9, 2),
             "encode_ms": round(enc_avg, 5), "decode_ms": round(dec_avg, 5),
+            "steps_per_s": round(1e3 / ms_step, 3),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 2), "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
                          "traffic": None if args.layers else _kernel_traffic(dom, w.name),
                          "alg_bytes_per_launch": dom_alg,
-                         "enc_frac": round(enc_alg / (enc_avg * 1e-3) / 1e9 / peak, 4),
-                         "dec_frac": round(dec_alg / (dec_avg * 1e-3) / 1e9 / peak, 4)},
-            "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": n_bf16,
-                    "d2h_bytes_per_step": n_bf16},
-            "gpu_launches": launches_per_step * args.steps,
+                         "enc_frac": round(P.enc_alg / (enc_avg * 1e-3) / 1e9 / peak, 4),
+                         "dec_frac": round(P.dec_alg / (dec_avg * 1e-3) / 1e9 / peak, 4)},
+            "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": P.h2d,
+                    "d2h_bytes_per_step": P.d2h},
+            "gpu_launches": P.launches * args.steps,
             "clocks": clk,
         }
         if not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_sample(w, G, seconds=args.cpu_seconds)
+            line["cpu_baseline"] = cpu_sample(w, P.G, seconds=args.cpu_seconds)
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()
