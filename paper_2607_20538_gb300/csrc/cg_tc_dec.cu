@@ -412,8 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
             // the previous TMA store of this warp has finished reading the staging block
             if (lane == 0) bulk_wait_read<0>();
             __syncwarp();
-#pragma unroll
-            for (int cc = 0; cc < 2; cc++) {
+            auto chunk = [&](int cc, const uint32_t (&d0)[32], const uint32_t (&d1)[32]) {
                 const int c = 2 * half + cc;  // 32-column chunk of the tile
                 // gauge group r = 32c / g (g >= 32) or several (g < 32, then nsub = 1)
                 const int r = (c * 32) / g;
@@ -429,16 +428,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                     const float m = __half2float(__ushort_as_half((unsigned short)(v >> 16)));
                     sk[k] = s;
                     ak[k] = m - kOff * s;
-                }
-                uint32_t d0[32], d1[32];
-                tmem_ld32(tacc + c * 32, d0);
-                if (nsub > 1) tmem_ld32(tacc + 128 + c * 32, d1);
-                tmem_wait_ld();
-                if (cc == 1) {
-                    // everything this warp needs from the buffer is in registers
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&M->accempty[buf]);
                 }
                 uint32_t o[16];
 #pragma unroll
@@ -472,6 +461,32 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
 #pragma unroll
                     for (int q = 0; q < 4; q++)
                         orow[c * 4 + q] = make_uint4(o[4 * q], o[4 * q + 1], o[4 * q + 2], o[4 * q + 3]);
+                }
+            };
+            auto release = [&]() {
+                // everything this warp needs from the buffer is in registers
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&M->accempty[buf]);
+            };
+            if (nsub == 1) {
+                // both chunks in flight before the single wait
+                uint32_t da[32], db[32];
+                tmem_ld32(tacc + (2 * half) * 32, da);
+                tmem_ld32(tacc + (2 * half + 1) * 32, db);
+                tmem_wait_ld();
+                release();
+                chunk(0, da, da);
+                chunk(1, db, db);
+            } else {
+#pragma unroll 1
+                for (int cc = 0; cc < 2; cc++) {
+                    uint32_t d0[32], d1[32];
+                    tmem_ld32(tacc + (2 * half + cc) * 32, d0);
+                    tmem_ld32(tacc + 128 + (2 * half + cc) * 32, d1);
+                    tmem_wait_ld();
+                    if (cc == 1) release();
+                    chunk(cc, d0, d1);
                 }
             }
             if (whole) {
