@@ -210,6 +210,30 @@ def _np_quantize(v, bits):
     return s16, m16, q
 
 
+@pytest.mark.parametrize("bits,blk", [(4, 64), (3, 32), (6, 128), (2, 64)])
+def test_planted_midpoints_hand_worked(bits, blk):
+    """fp16 round-half-even on exact midpoints of the scale (max - min) / qmax and of the
+    zero (an fp16 subnormal midpoint), exact half-integer codes, constant and zero blocks
+    (Sec. 4.3 quantizer): the values worked out by hand in planted.py."""
+    from planted import N_KINDS, expected_scale_zero, planted_rows
+    w = _wl(T=12, d=128, group=128, block=blk, bits=bits)
+    qmax = 2 ** bits - 1
+    x, kind = planted_rows(w, np.random.default_rng(bits))
+    r = oracle.encode(w.shape, w.params, x, synth.gauges(w, "identity"))
+    sm = r["scales"].reshape(kind.shape + (2,))
+    for k in range(N_KINDS):
+        es, em = expected_scale_zero(k, qmax)
+        if es is not None:
+            assert (sm[..., 0][kind == k] == es).all(), k
+        if em is not None:
+            assert (sm[..., 1][kind == k] == em).all(), k
+    q = oracle.unpack(r["codes"], x.size, bits).reshape(x.shape)
+    per_elem = np.repeat(kind, blk, axis=-1)
+    xv = _f32(x)
+    np.testing.assert_array_equal(q[per_elem == 0], np.rint(xv[per_elem == 0]))
+    assert (q[(per_elem == 2) | (per_elem == 3)] == 0).all()
+
+
 @pytest.mark.parametrize("bits,blk,g", [(4, 16, 8), (3, 32, 32), (6, 32, 16), (2, 8, 8), (8, 64, 64)])
 def test_identity_gauge_is_bare_backend(bits, blk, g):
     """Sec. 4.3: the identity gauge compresses the raw cache, so encode must equal the
