@@ -8,13 +8,16 @@
 // D[token][i] = sum_j A[token][j] B[i][j] with B = G^T (two bf16 terms) takes three MMA
 // passes (hi·hi, hi·lo, lo·hi; the lo·lo term is below 2^-16 relative).
 //
-// Persistent warp-specialized kernel, one CTA per SM, 10 warps:
+// Persistent warp-specialized kernel, one CTA per SM, 14 warps:
 //   warp 0      bulk copy of a group's code streams (128 x 16*bits bytes) and its 128 scales;
-//   warp 1      MMA issuer (24 MMAs per tile, fp32 accumulators, two TMEM buffers);
-//   warps 2..5  one gauge-space channel per thread: unpack, dequantize, split, store the
-//               channel's column of the A tile; at a gauge change they build G^T's split
-//               (full K, block-diagonal for g < 128);
-//   warps 6..9  one token row per thread: accumulator -> bf16 -> global.
+//   warp 1      MMA issuer (24 MMAs per tile, each one gauge group wide, fp32 accumulators,
+//               two TMEM buffers);
+//   warps 2..9  one gauge-space channel and 64 of its tokens per thread (warps 2..5 the
+//               first 64 tokens, 6..9 the others): unpack, dequantize, split, store that
+//               part of the channel's column of the A tile; at a gauge change warps 2..5
+//               build G^T's split (full K for g = 128; for smaller groups the diagonal
+//               blocks packed into one 64-column tile, one MMA chain per group);
+//   warps 10..13 one token row per thread: accumulator -> bf16 -> global.
 #include <cuda_bf16.h>
 
 #include "cg_sm100.cuh"
@@ -28,8 +31,8 @@ using namespace sm100;
 using tc::kD;
 using tc::kWaitLimitNs;
 
-constexpr int kThreads = 320;
-constexpr int kEpiWarp0 = 6;
+constexpr int kThreads = 448;
+constexpr int kEpiWarp0 = 10;
 constexpr int kATerm = 128 * kD * 2;  // one bf16 term of a 128 x 128 tile
 constexpr int kAStages = 2;
 constexpr int kSegBufs = 4;
@@ -81,6 +84,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
     const int g = a.g;
+    const int gb = g < 16 ? 16 : g;  // MMA width: one gauge group (two for g = 8)
+    // G^T split: full K for g = 128, else the groups' diagonal blocks packed into one
+    // 64-column tile per term (rows of a group at its own channels)
+    const uint32_t bsz = g == 128 ? 32768u : 16384u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
@@ -91,10 +98,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
     if (threadIdx.x == 0) {
         for (int i = 0; i < kCStages; i++) {
             mbar_init(&M->cfull[i], 1);
-            mbar_init(&M->cempty[i], 4);
+            mbar_init(&M->cempty[i], 8);
         }
         for (int i = 0; i < kAStages; i++) {
-            mbar_init(&M->afull[i], 4);
+            mbar_init(&M->afull[i], 8);
             mbar_init(&M->aempty[i], 1);
         }
         for (int i = 0; i < 2; i++) {
@@ -150,8 +157,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && my_tiles > 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, 128);
+            const uint32_t idesc = idesc_bf16_f32(128, gb);
             const uint64_t bdesc = sdesc_sw128(smem_u32(bsplit));
+            // the tile's 24 MMAs (3 term pairs x 8 K-steps of 16 over the groups): D column,
+            // A and B byte offsets (in 16-byte units), accumulate bits
+            uint32_t q_d[kMma], q_a[kMma], q_b[kMma], q_acc = 0;
+#pragma unroll
+            for (int q = 0; q < kMma; q++) {
+                const int pair = q >> 3, qq = q & 7;  // pairs: (A hi, B hi), (A hi, B lo), (A lo, B hi)
+                const uint32_t ta = pair == 2 ? 1u : 0u, tb = pair == 1 ? 1u : 0u;
+                const int per = gb >> 4;  // K-steps per group
+                const int r = qq / per, ks = qq - r * per;
+                const int k0 = r * gb + ks * 16;
+                q_d[q] = (uint32_t)(r * gb);
+                q_a[q] = (ta * kATerm + (uint32_t)((k0 >> 6) * 16384 + (k0 & 63) * 2)) >> 4;
+                q_b[q] = (tb * bsz + (uint32_t)((g == 128 ? (k0 >> 6) * 16384 : r * gb * 128) + (k0 & 63) * 2)) >> 4;
+                q_acc |= (pair > 0 || ks > 0 ? 1u : 0u) << q;
+            }
             int64_t cur = -1;
             int committed = 0;
             tc::TileIter it;
@@ -175,13 +197,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 const uint64_t adesc = sdesc_sw128(smem_u32(atiles + ab * 2 * kATerm));
                 const uint32_t d_base = tmem + buf * 128;
 #pragma unroll
-                for (int q = 0; q < kMma; q++) {
-                    const int pair = q >> 3, ks = q & 7;  // pairs: (A hi, B hi), (A hi, B lo), (A lo, B hi)
-                    const uint32_t ta = pair == 2 ? 1u : 0u, tb = pair == 1 ? 1u : 0u;
-                    const uint32_t koff = (uint32_t)((ks >> 2) * 16384 + (ks & 3) * 32);  // K = 16 ks
-                    mma_bf16(d_base, adesc + ((ta * kATerm + koff) >> 4), bdesc + ((tb * 32768u + koff) >> 4), idesc,
-                             q > 0 ? 1u : 0u);
-                }
+                for (int q = 0; q < kMma; q++)
+                    mma_bf16(d_base + q_d[q], adesc + q_a[q], bdesc + q_b[q], idesc, (q_acc >> q) & 1u);
                 mma_commit(&M->accfull[buf]);
                 mma_commit(&M->aempty[ab]);
                 const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
@@ -196,14 +213,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
         }
     } else if (warp < kEpiWarp0) {
         // ------------------------------------------------------------ unpack + dequantize
-        const int ch = (warp - 2) * 32 + lane;  // gauge-space channel of this thread
+        const int ch = ((warp - 2) & 3) * 32 + lane;  // gauge-space channel of this thread
+        const int half = (warp - 2) >> 2;             // its tokens: 64 half .. 64 half + 63
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
         it.init(a, S, t_begin);
         for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
             const tc::TileInfo ti = it.info(a);
-            if (ti.seg != cur) {
+            if (ti.seg != cur && half == 0) {
                 const int64_t ls = ti.seg - seg0;
                 if (nconv > 0) {
                     const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
@@ -228,9 +246,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                         lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
                     }
                     const int k = r * g + j;
-                    const uint32_t off = (k >> 6) * 16384 + sw128_offset(n, k & 63);
+                    const uint32_t off = (g == 128 ? (k >> 6) * 16384 : 0) + sw128_offset(n, k & 63);
                     *reinterpret_cast<uint4*>(bsplit + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
-                    *reinterpret_cast<uint4*>(bsplit + 32768 + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+                    *reinterpret_cast<uint4*>(bsplit + bsz + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                 }
                 fence_proxy_async_smem();
                 __syncwarp();
@@ -246,25 +264,24 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 break;
             }
             const unsigned char* stage = cst + st * kCStageBytes;
-            uint32_t w[4 * BITS + 1];
+            // this thread's 64 codes: 8 * BITS bytes of the channel stream
+            uint32_t w[2 * BITS + 1];
 #pragma unroll
             for (int q = 0; q < BITS; q++) {
-                const uint4 v = reinterpret_cast<const uint4*>(stage + ch * kStreamBytes)[q];
-                w[4 * q] = v.x;
-                w[4 * q + 1] = v.y;
-                w[4 * q + 2] = v.z;
-                w[4 * q + 3] = v.w;
+                const uint2 v = reinterpret_cast<const uint2*>(stage + ch * kStreamBytes + half * 8 * BITS)[q];
+                w[2 * q] = v.x;
+                w[2 * q + 1] = v.y;
             }
-            w[4 * BITS] = 0;
+            w[2 * BITS] = 0;
             const uint32_t sz = reinterpret_cast<const uint32_t*>(stage + 128u * kStreamBytes)[ch];
             const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
             const float m = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
             // column ch of the token-major A tile: token t at row t (128-byte swizzle)
-            unsigned char* ahi = atiles + ab * 2 * kATerm + (ch >> 6) * 16384 + (ch & 7) * 2;
+            unsigned char* ahi = atiles + ab * 2 * kATerm + (ch >> 6) * 16384 + (ch & 7) * 2 + half * 64 * 128;
             unsigned char* alo = ahi + kATerm;
             const int cu = (ch & 63) >> 3;
 #pragma unroll
-            for (int t = 0; t < 128; t++) {
+            for (int t = 0; t < 64; t++) {
                 const int p = t * BITS;
                 uint32_t v = w[p >> 5] >> (p & 31);
                 if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));

@@ -44,6 +44,8 @@ CASES = {
     "kivi4_g128_blk128": _wl(backend=1, group=128, bits=4, block=128, residual=16, T=400),
     "kivi3_g32_blk128_B3_R0": _wl(backend=1, group=32, bits=3, block=128, residual=0, T=300, B=3),
     "kivi8_g64_blk128": _wl(backend=1, group=64, bits=8, block=128, residual=128, T=520, L=1, H=3),
+    "kivi3_g8_blk128_R0": _wl(backend=1, group=8, bits=3, block=128, residual=0, T=256),
+    "kivi4_g16_blk128": _wl(backend=1, group=16, bits=4, block=128, residual=32, T=300),
     "none_g128": _wl(backend=2, group=128, T=260),
     "none_g8_d64": _wl(backend=2, d=64, group=8, T=33),
 }
