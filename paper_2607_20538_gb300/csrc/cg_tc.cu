@@ -19,9 +19,12 @@
 // products; include/codecgauge.h). For every output channel i the converter bounds
 // |z~_i - z_i| / ||x_group||_2 by
 //     e_i = (c_order + c_tc) ||G_i||_2 + ||G_i - sum of split terms||_2,
-// c_order = (1 + log2 g) u the rounding bound of the fixed order, c_tc = (n_mma + 2) u a
-// bound on the tensor-core fp32 accumulation over its n_mma K=16 steps (the measured
-// error stays several times below it), and the exact residual of the split. The epilogue
+// c_order = (1 + log2 g) u the rounding bound of the fixed order, c_tc a bound on the
+// tensor-core fp32 accumulation, and the exact residual of the split. The MMAs accumulate
+// the split's two small terms first (partial sums below 2^-8 of ||G_i|| ||x||, 2 n_hi
+// K-steps) and the leading term last (n_hi = K / 16 steps), so c_tc = (n_hi + 4 + 2 n_hi /
+// 128) u, 4 u covering the rounding inside each MMA and of the result; the measured
+// |z~ - Gx| stays below 2.4 u ||G_i|| ||x|| (g = 32 and 128; random, Hadamard and DCT gauges). The epilogue
 // turns it into E per block. A block's fp16 scale and zero are monotone functions of its
 // (max, min); when every (max, min) within E of the approximate ones gives the same fp16
 // results they are taken directly, otherwise the candidate extremes are recomputed
@@ -338,7 +341,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         // ------------------------------------------------------------ gauge converter
         const int lg = 31 - __clz(g);
         const float c_order = (float)(1 + lg) * kU * 1.01f;
-        const float c_tc = (float)(npass * ((KEYS ? 128 : gb) / 16) + 2) * kU;
+        // the split's two small terms are accumulated first (their partial sums stay below
+        // 2^-8 of the group's scale), so the accumulation error is dominated by the n_hi
+        // K-steps of the leading term; 4 u covers the rounding inside each MMA and of the result
+        const int n_hi = (KEYS ? 128 : gb) / 16;
+        const float c_tc = ((float)n_hi + 4.0f + (float)((npass - 1) * n_hi) * (1.0f / 128.0f)) * kU;
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
