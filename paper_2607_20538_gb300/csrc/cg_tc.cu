@@ -2,18 +2,20 @@
 // rotation (Sec. 3, Z = G X) fused with the block-uniform quantizer of Sec. 4.3 (one range
 // per block of `block` channels of a token), also used for KIVI value rows.
 //
-// Persistent warp-specialized kernel, one CTA per SM, 11 warps:
+// Persistent warp-specialized kernel, one CTA per SM, 15 warps:
 //   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte
 //               swizzle) into a 4-stage ring;
 //   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group,
 //               one MMA chain per group block), G split into three bf16 terms (hi + lo +
 //               lo2, exact for normal fp32 values); fp32 accumulators in tensor memory,
-//               four buffers (the MMA runs up to two tiles ahead of each warpgroup);
+//               four buffers (the MMA runs one tile ahead of the three warpgroups);
 //   warp 2      gauge converter: at each gauge change builds the bf16 split operand and
 //               the per-block error coefficients of the new gauge set;
-//   warps 3..10 two epilogue warpgroups; warpgroup k takes every other tile; one thread
-//               per token row (= TMEM lane): block min/max, fp16 scale/zero, codes,
-//               packing, stores.
+//   warps 3..14 three epilogue warpgroups; warpgroup k takes tiles i = k (mod 3); one
+//               thread per token row (= TMEM lane): block min/max, fp16 scale/zero, codes,
+//               packing, stores. The number of quantization blocks per row is a template
+//               parameter, so the per-block state of a row takes only the registers it
+//               needs (128 per thread for 15 warps).
 //
 // Exactness. The library defines z as a fixed-order fp32 sum (pairwise summation of the
 // products; include/codecgauge.h). For every output channel i the converter bounds
@@ -52,9 +54,9 @@ using tc::kWaitLimitNs;
 
 constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
-constexpr int kThreads = 352;
+constexpr int kThreads = 480;
 constexpr int kEpiWarp0 = 3;
-constexpr int kQCap = 32;             // repair jobs per warp and round
+constexpr int kQCap = 24;             // repair jobs per warp and round
 constexpr int kAcc = 4;               // accumulator buffers in tensor memory
 constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
@@ -64,8 +66,8 @@ constexpr float kMagic = 12582912.0f; // 1.5 * 2^23: adding it rounds to an inte
 struct EncSmem {
     static constexpr uint32_t stages = 0;
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
-    static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 8 warps x kQCap x 8 B
-    static constexpr uint32_t misc = queue + 8 * kQCap * 8;
+    static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 12 warps x kQCap x 8 B
+    static constexpr uint32_t misc = queue + 12 * kQCap * 8;
     static constexpr uint32_t total = misc + 384;  // base is 1024-aligned (checked in-kernel)
 };
 
@@ -196,7 +198,7 @@ __device__ __forceinline__ void patch_code(uint8_t* rowp, int bit, uint32_t q) {
 // KEYS = true: KIVI keys (Sec. 4.3, per-channel ranges over a 128-token group): the MMA
 // operands are swapped, D[channel][token] = G x^T, so a thread owns one channel's 128
 // tokens, which form its block and its packed code stream.
-template <int BITS, bool KEYS>
+template <int BITS, bool KEYS, int NBK>
 __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_constant__ CUtensorMap xmap,
                                                                  const EncParams P) {
     extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -213,9 +215,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
-    const int g = a.g, blk = a.blk, npass = kNPass;
+    const int g = a.g, npass = kNPass;
+    constexpr int blk = kD / NBK;  // quantization block: NBK blocks per row
     const int gb = g < 16 ? 16 : g;
-    const int nbk = kD / blk;
+    constexpr int nbk = NBK;
     // gauge operand layout: full K = 128 (block-diagonal for g < 128) for keys and g = 128,
     // else one g-wide K block per group in a 64-column tile
     const bool fullk = KEYS || g == 128;
@@ -461,7 +464,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         }
     } else {
         // ------------------------------------------------------------ epilogue warpgroups
-        const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup: tiles i = wg (mod 2)
+        const int wg = (warp - kEpiWarp0) >> 2;       // warpgroup: tiles i = wg (mod 3)
         const int q4 = warp & 3;                      // TMEM lane quadrant of this warp
         const int row = q4 * 32 + lane;               // TMEM lane: token (rows) or channel (keys)
         const int qw = warp - kEpiWarp0;              // job queue of this warp
@@ -479,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         int32_t flag = 0;
         tc::TileIter it;
         it.init(a, S, t_begin + wg);
-        for (int i = wg; i < my_tiles; i += 2, it.step(a, 2)) {
+        for (int i = wg; i < my_tiles; i += 3, it.step(a, 3)) {
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
             const int st = i % kStages, buf = i % kAcc;
@@ -887,15 +890,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     }
 }
 
-template <int BITS, bool KEYS>
-cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
+template <int BITS, bool KEYS, int NBK>
+cudaError_t launch_encode_nbk(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
     const size_t smem = EncSmem::total;
     cudaError_t e =
-        cudaFuncSetAttribute(tc_encode_kernel<BITS, KEYS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(tc_encode_kernel<BITS, KEYS, NBK>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
-    tc_encode_kernel<BITS, KEYS><<<(unsigned)grid, kThreads, smem, st>>>(map, P);
+    tc_encode_kernel<BITS, KEYS, NBK><<<(unsigned)grid, kThreads, smem, st>>>(map, P);
     return cudaGetLastError();
+}
+
+// keys: one block (the 128-token group) per channel; rows: 128 / block blocks per row
+template <int BITS, bool KEYS>
+cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
+    if constexpr (KEYS) {
+        return launch_encode_nbk<BITS, KEYS, 1>(P, map, st);
+    } else {
+        if (P.a.blk == 128) return launch_encode_nbk<BITS, KEYS, 1>(P, map, st);
+        if (P.a.blk == 64) return launch_encode_nbk<BITS, KEYS, 2>(P, map, st);
+        return launch_encode_nbk<BITS, KEYS, 4>(P, map, st);
+    }
 }
 
 template <bool KEYS>
