@@ -15,7 +15,8 @@
 //               thread per token row (= TMEM lane): block min/max, fp16 scale/zero, codes,
 //               packing, stores. The number of quantization blocks per row is a template
 //               parameter, so the per-block state of a row takes only the registers it
-//               needs (128 per thread for 15 warps).
+//               needs (128 per thread for 15 warps); codes are packed into the output
+//               words as they are produced.
 //
 // Exactness. The library defines z as a fixed-order fp32 sum (pairwise summation of the
 // products; include/codecgauge.h). For every output channel i the converter bounds
@@ -761,18 +762,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const float r = pick4(rinv, bk), cc = pick4(c0, bk), lm = pick4(lim, bk);
                 const bool fst = (fast >> bk) & 1;
                 const bool lv = (live >> bk) & 1;
-                uint32_t qv[32];
                 float dmax = 0.0f;
+                uint32_t words[BITS];
+#pragma unroll
+                for (int w = 0; w < BITS; w++) words[w] = 0;
+                // code k into the packed little-endian stream of this 32-code chunk
+                auto put = [&](int k, uint32_t y) {
+                    const uint32_t q = y & (uint32_t)qmax;
+                    const int bit = k * BITS;
+                    words[bit >> 5] |= q << (bit & 31);
+                    if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
+                };
                 if (fst && lm > 1.0f) {
 #pragma unroll
-                    for (int k = 0; k < 32; k++) qv[k] = __float_as_uint(fmaf(__uint_as_float(v[k]), r, cc) + kMagic);
+                    for (int k = 0; k < 32; k++) put(k, __float_as_uint(fmaf(__uint_as_float(v[k]), r, cc) + kMagic));
                 } else if (fst) {
 #pragma unroll
                     for (int k = 0; k < 32; k++) {
                         const float t = fmaf(__uint_as_float(v[k]), r, cc);
                         const float y = t + kMagic;
                         dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
-                        qv[k] = __float_as_uint(y);
+                        put(k, __float_as_uint(y));
                     }
                 } else {
 #pragma unroll
@@ -781,18 +791,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         t = fminf(fmaxf(t, 0.0f), qmaxf);
                         const float y = t + kMagic;
                         dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
-                        qv[k] = lv ? __float_as_uint(y) : 0u;
+                        put(k, lv ? __float_as_uint(y) : 0u);
                     }
-                }
-                uint32_t words[BITS];
-#pragma unroll
-                for (int w = 0; w < BITS; w++) words[w] = 0;
-#pragma unroll
-                for (int k = 0; k < 32; k++) {
-                    const uint32_t q = qv[k] & (uint32_t)qmax;
-                    const int bit = k * BITS;
-                    words[bit >> 5] |= q << (bit & 31);
-                    if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
                 }
                 if (valid) {
                     uint32_t* dst = reinterpret_cast<uint32_t*>(crow) + c * BITS;
