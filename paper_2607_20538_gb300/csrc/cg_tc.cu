@@ -762,7 +762,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const float r = pick4(rinv, bk), cc = pick4(c0, bk), lm = pick4(lim, bk);
                 const bool fst = (fast >> bk) & 1;
                 const bool lv = (live >> bk) & 1;
-                float dmax = 0.0f;
                 uint32_t words[BITS];
 #pragma unroll
                 for (int w = 0; w < BITS; w++) words[w] = 0;
@@ -773,24 +772,18 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     words[bit >> 5] |= q << (bit & 31);
                     if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
                 };
+                uint32_t mk = 0;  // values within mu of a rounding boundary (bit k: column 32c + k)
                 if (fst && lm > 1.0f) {
 #pragma unroll
                     for (int k = 0; k < 32; k++) put(k, __float_as_uint(fmaf(__uint_as_float(v[k]), r, cc) + kMagic));
-                } else if (fst) {
-#pragma unroll
-                    for (int k = 0; k < 32; k++) {
-                        const float t = fmaf(__uint_as_float(v[k]), r, cc);
-                        const float y = t + kMagic;
-                        dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
-                        put(k, __float_as_uint(y));
-                    }
                 } else {
+                    // clamping before the rounding gives the same code as clamping after it
 #pragma unroll
-                    for (int k = 0; k < 32; k++) {
+                    for (int k = 31; k >= 0; k--) {
                         float t = fmaf(__uint_as_float(v[k]), r, cc);
                         t = fminf(fmaxf(t, 0.0f), qmaxf);
                         const float y = t + kMagic;
-                        dmax = fmaxf(dmax, fabsf(t - (y - kMagic)));
+                        mk = __funnelshift_l(__float_as_uint(__fsub_rn(lm, fabsf(t - (y - kMagic)))), mk, 1);
                         put(k, lv ? __float_as_uint(y) : 0u);
                     }
                 }
@@ -808,17 +801,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         for (int w = 0; w < BITS; w++) dst[w] = words[w];
                     }
                 }
-                if (valid && lv && dmax > lm) {
-                    uint32_t mk = 0;
-#pragma unroll
-                    for (int k = 0; k < 32; k++) {
-                        float t = fmaf(__uint_as_float(v[k]), r, cc);
-                        if (!fst) t = fminf(fmaxf(t, 0.0f), qmaxf);
-                        const float y = t + kMagic;
-                        if (fabsf(t - (y - kMagic)) > lm) mk |= 1u << k;
-                    }
-                    set4(am, c, mk);
-                }
+                if (valid && lv) set4(am, c, mk);
             }
             bool pend = (am[0] | am[1] | am[2] | am[3]) != 0;
             while (__any_sync(0xffffffffu, pend)) {
