@@ -547,7 +547,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         gm[rr] = fmaxf(gm[rr], __shfl_xor_sync(0xffffffffu, gm[rr], off));
                 bs[0] = pick4(gm, row / g);  // fmaxf keeps a NaN out; non-finite input is flagged above
             }
-#pragma unroll 4
+            // unroll depth measured per block count (code size against load parallelism)
+            constexpr int kNormUnroll = NBK == 2 ? 8 : (NBK == 4 ? 2 : 4);
+#pragma unroll kNormUnroll
             for (int c8 = 0; c8 < (KEYS ? 0 : 16); c8++) {
                 const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
                                                                  (((c8 & 7) ^ (row & 7)) << 4));
