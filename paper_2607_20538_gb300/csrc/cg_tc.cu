@@ -135,7 +135,7 @@ __device__ __forceinline__ void bound_range(int bk, int g, int blk, int& lo, int
 // their pairwise sum, and the team combines its partial sums with xor-shuffles, which
 // follows the same pairwise tree. Each lane loads the operands of kSlots values before any
 // arithmetic, so one memory round trip serves kSlots x (32 / T) values.
-constexpr int kSlots = 4;
+template <int kSlots>
 __device__ __noinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned char* stage, const float* Gf, int g,
                                       int lane) {
     const int lgT = 29 - __clz(g);  // log2(g / 4); g in {8, ..., 128}
@@ -220,6 +220,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     constexpr int blk = kD / NBK;  // quantization block: NBK blocks per row
     const int gb = g < 16 ? 16 : g;
     constexpr int nbk = NBK;
+    // values per lane and memory round trip in the exact recompute (measured: 4 with two
+    // blocks per row, the 8B-shaped cache; 2 with one or four)
+    constexpr int kJobSlots = NBK == 2 ? 4 : 2;
     // gauge operand layout: full K = 128 (block-diagonal for g < 128) for keys and g = 128,
     // else one g-wide K block per group in a 64-column tile
     const bool fullk = KEYS || g == 128;
@@ -683,7 +686,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         }
                     }
                     __syncwarp();
-                    run_jobs(qjob, min(total, kQCap), stg, Gf, g, lane);
+                    run_jobs<kJobSlots>(qjob, min(total, kQCap), stg, Gf, g, lane);
                     __syncwarp();
                     // the same candidates in the same order: fold the exact values in
                     slot = base;
@@ -828,7 +831,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                     }
                 }
                 __syncwarp();
-                run_jobs(qjob, min(total, kQCap), stg, Gf, g, lane);
+                run_jobs<kJobSlots>(qjob, min(total, kQCap), stg, Gf, g, lane);
                 __syncwarp();
                 slot = base;
 #pragma unroll 1
