@@ -19,7 +19,9 @@
 //               in shared memory (128-byte swizzle) and writes it with one TMA tile store.
 //               Each thread loads the next tile's block scales one tile ahead.
 // With the scale and zero of a block constant along the token, dequantization commutes
-// with the rotation, so the integer codes go through the tensor cores unscaled.
+// with the rotation, so the integer codes go through the tensor cores unscaled. The number
+// of sub-block accumulators is a template parameter, so each kernel holds only its own
+// epilogue.
 #include <cuda_bf16.h>
 
 #include "cg_sm100.cuh"
@@ -118,7 +120,7 @@ __device__ __forceinline__ void unpack_row(const uint32_t* w, uint4 (&out)[16]) 
     }
 }
 
-template <int BITS>
+template <int BITS, int NSUB>
 __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_constant__ CUtensorMap omap,
                                                                  const DecParams P) {
     using SL = DecSmem<BITS>;
@@ -135,7 +137,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
 
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
-    const int g = a.g, blk = a.blk, nsub = P.nsub;
+    const int g = a.g, blk = a.blk;
+    constexpr int nsub = NSUB;  // accumulators per gauge group
     const int gb = g < 16 ? 16 : g;
     const uint32_t bsz = (g == 128) ? 32768u : 16384u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -509,14 +512,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
     }
 }
 
-template <int BITS>
-cudaError_t launch_dec(const DecParams& P, const CUtensorMap& omap, cudaStream_t st) {
+template <int BITS, int NSUB>
+cudaError_t launch_dec_ns(const DecParams& P, const CUtensorMap& omap, cudaStream_t st) {
     const size_t smem = DecSmem<BITS>::total + 1024;
-    cudaError_t e = cudaFuncSetAttribute(tc_decode_kernel<BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e =
+        cudaFuncSetAttribute(tc_decode_kernel<BITS, NSUB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t grid = P.S.n_tiles < tc::num_sms() ? P.S.n_tiles : tc::num_sms();
-    tc_decode_kernel<BITS><<<(unsigned)grid, kThreads, smem, st>>>(omap, P);
+    tc_decode_kernel<BITS, NSUB><<<(unsigned)grid, kThreads, smem, st>>>(omap, P);
     return cudaGetLastError();
+}
+
+template <int BITS>
+cudaError_t launch_dec(const DecParams& P, const CUtensorMap& omap, cudaStream_t st) {
+    return P.nsub > 1 ? launch_dec_ns<BITS, 2>(P, omap, st) : launch_dec_ns<BITS, 1>(P, omap, st);
 }
 
 }  // namespace
