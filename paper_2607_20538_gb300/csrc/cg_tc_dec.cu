@@ -482,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 chunk(0, da, da);
                 chunk(1, db, db);
             } else {
-#pragma unroll 1
+#pragma unroll
                 for (int cc = 0; cc < 2; cc++) {
                     uint32_t d0[32], d1[32];
                     tmem_ld32(tacc + (2 * half + cc) * 32, d0);
