@@ -160,6 +160,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
            | ((uint32_t)(N >> 3) << 17)       // N / 8
            | ((uint32_t)(M >> 4) << 24);      // M / 16
 }
+// Bit of the instruction descriptor that makes A MN-major (transposed).
+constexpr uint32_t kIdescAMnMajor = 1u << 15;
 
 // Shared-memory matrix descriptor for a K-major operand stored in the 128-byte swizzle
 // layout: rows of 128 B (64 bf16), 8-row atoms of 1024 B (stride byte offset), the tile
@@ -171,6 +173,19 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
     d |= (uint64_t)(1024u >> 4) << 32;  // stride byte offset: 8 rows x 128 B
     d |= (uint64_t)1 << 46;             // descriptor version for sm_100
     d |= (uint64_t)2 << 61;             // swizzle mode: 128 B
+    return d;
+}
+
+// Shared-memory descriptor of an MN-major operand in the 128-byte swizzle layout: atoms of
+// 8 K-rows x 64 MN-elements (1024 B, rows of 128 B, 16-byte chunks XOR-swizzled by the row),
+// `lbo` bytes between atoms along MN, `sbo` bytes between atoms along K.
+__device__ __forceinline__ uint64_t sdesc_sw128_mn(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
     return d;
 }
 

@@ -4,7 +4,9 @@
 // A key group stores, per gauge-space channel, a stream of 128 token codes with one scale
 // and zero, so the scale varies along the contraction index of Xhat = G^T Zhat and cannot
 // be applied after the MMA. The unpackers therefore dequantize, zhat = q s + m in fp32, and
-// write zhat as two bf16 terms (hi + lo, 16 significant bits) into a token-major A tile;
+// write zhat as two bf16 terms (hi + lo, 16 significant bits) into an A tile that the MMA
+// reads MN-major (tokens contiguous per channel, as the code streams are), so a thread
+// stores 8 tokens of its channel at a time;
 // D[token][i] = sum_j A[token][j] B[i][j] with B = G^T (two bf16 terms) takes three MMA
 // passes (hi·hi, hi·lo, lo·hi; the lo·lo term is below 2^-16 relative).
 //
@@ -14,7 +16,7 @@
 //               two TMEM buffers);
 //   warps 2..9  one gauge-space channel and 64 of its tokens per thread (warps 2..5 the
 //               first 64 tokens, 6..9 the others): unpack, dequantize, split, store that
-//               part of the channel's column of the A tile; at a gauge change warps 2..5
+//               part of the channel's K-row of the A tile; at a gauge change warps 2..5
 //               build G^T's split (full K for g = 128; for smaller groups the diagonal
 //               blocks packed into one 64-column tile, one MMA chain per group);
 //   warps 10..13 one token row per thread: accumulator -> bf16 -> global.
@@ -157,7 +159,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0 && my_tiles > 0) {
-            const uint32_t idesc = idesc_bf16_f32(128, gb);
+            const uint32_t idesc = idesc_bf16_f32(128, gb) | kIdescAMnMajor;  // A read MN-major
             const uint64_t bdesc = sdesc_sw128(smem_u32(bsplit));
             // the tile's 24 MMAs (3 term pairs x 8 K-steps of 16 over the groups): D column,
             // A and B byte offsets (in 16-byte units), accumulate bits
@@ -170,7 +172,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 const int r = qq / per, ks = qq - r * per;
                 const int k0 = r * gb + ks * 16;
                 q_d[q] = (uint32_t)(r * gb);
-                q_a[q] = (ta * kATerm + (uint32_t)((k0 >> 6) * 16384 + (k0 & 63) * 2)) >> 4;
+                q_a[q] = (ta * kATerm + (uint32_t)((k0 >> 3) * 1024)) >> 4;  // K-step: two 8-channel atoms
                 q_b[q] = (tb * bsz + (uint32_t)((g == 128 ? (k0 >> 6) * 16384 : r * gb * 128) + (k0 & 63) * 2)) >> 4;
                 q_acc |= (pair > 0 || ks > 0 ? 1u : 0u) << q;
             }
@@ -194,7 +196,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                     break;
                 }
                 tc_fence_after();
-                const uint64_t adesc = sdesc_sw128(smem_u32(atiles + ab * 2 * kATerm));
+                const uint64_t adesc = sdesc_sw128_mn(smem_u32(atiles + ab * 2 * kATerm), 16384u, 1024u);
                 const uint32_t d_base = tmem + buf * 128;
 #pragma unroll
                 for (int q = 0; q < kMma; q++)
@@ -276,21 +278,33 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
             const uint32_t sz = reinterpret_cast<const uint32_t*>(stage + 128u * kStreamBytes)[ch];
             const float s = __half2float(__ushort_as_half((unsigned short)(sz & 0xffffu)));
             const float m = __half2float(__ushort_as_half((unsigned short)(sz >> 16)));
-            // column ch of the token-major A tile: token t at row t (128-byte swizzle)
-            unsigned char* ahi = atiles + ab * 2 * kATerm + (ch >> 6) * 16384 + (ch & 7) * 2 + half * 64 * 128;
+            // MN-major A tile: channel ch is K-row (ch & 7) of atom (half, ch >> 3); its 64 tokens
+            // are 8 chunks of 8 (16 bytes), chunk c stored at position c ^ (ch & 7)
+            unsigned char* ahi = atiles + ab * 2 * kATerm + half * 16384 + (ch >> 3) * 1024 + (ch & 7) * 128;
             unsigned char* alo = ahi + kATerm;
-            const int cu = (ch & 63) >> 3;
 #pragma unroll
-            for (int t = 0; t < 64; t++) {
-                const int p = t * BITS;
-                uint32_t v = w[p >> 5] >> (p & 31);
-                if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
-                const float z = fmaf((float)(v & ((1u << BITS) - 1u)), s, m);
-                const __nv_bfloat16 h = __float2bfloat16_rn(z);
-                const __nv_bfloat16 l = __float2bfloat16_rn(z - __bfloat162float(h));
-                const uint32_t o = t * 128 + ((cu ^ (t & 7)) << 4);
-                *reinterpret_cast<__nv_bfloat16*>(ahi + o) = h;
-                *reinterpret_cast<__nv_bfloat16*>(alo + o) = l;
+            for (int c = 0; c < 8; c++) {
+                uint32_t hi[4], lo[4];
+#pragma unroll
+                for (int e = 0; e < 4; e++) {
+                    float z2[2];
+#pragma unroll
+                    for (int u = 0; u < 2; u++) {
+                        const int t = 8 * c + 2 * e + u;
+                        const int p = t * BITS;
+                        uint32_t v = w[p >> 5] >> (p & 31);
+                        if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
+                        z2[u] = fmaf((float)(v & ((1u << BITS) - 1u)), s, m);
+                    }
+                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(z2[0], z2[1]);
+                    const float2 hf = __bfloat1622float2(h2);
+                    const __nv_bfloat162 l2 = __floats2bfloat162_rn(z2[0] - hf.x, z2[1] - hf.y);
+                    hi[e] = *reinterpret_cast<const uint32_t*>(&h2);
+                    lo[e] = *reinterpret_cast<const uint32_t*>(&l2);
+                }
+                const uint32_t o = (uint32_t)((c ^ (ch & 7)) << 4);
+                *reinterpret_cast<uint4*>(ahi + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+                *reinterpret_cast<uint4*>(alo + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
             }
             fence_proxy_async_smem();
             __syncwarp();
