@@ -175,6 +175,16 @@ __device__ __noinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned cha
     }
 }
 
+// The constant part of a packed word built from y = 0x4B400000 + q: the wrapping sum of
+// 0x4B400000 << s over the codes of a 32-code chunk that start in word w.
+template <int BITS>
+__host__ __device__ constexpr uint32_t pack_bias(int w) {
+    uint32_t k = 0;
+    for (int c = 0; c < 32; c++)
+        if ((c * BITS) >> 5 == w) k += 0x4B400000u << ((c * BITS) & 31);
+    return k;
+}
+
 __device__ __forceinline__ uint32_t scale16(float mx, float mn, float qmax) {
     return f2h_bits(__fdiv_rn(__fsub_rn(mx, mn), qmax));
 }
@@ -771,11 +781,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 #pragma unroll
                 for (int w = 0; w < BITS; w++) words[w] = 0;
                 // code k into the packed little-endian stream of this 32-code chunk
+                // y = kMagic + q has the bit pattern 0x4B400000 + q. Widths that straddle words
+                // (3, 6 bits) measure faster with a wrapping sum of y << s per word, less the
+                // constant sum of 0x4B400000 << s; the others mask and OR the codes in.
+                constexpr bool kBiasPack = BITS == 3 || BITS == 6;
                 auto put = [&](int k, uint32_t y) {
-                    const uint32_t q = y & (uint32_t)qmax;
                     const int bit = k * BITS;
-                    words[bit >> 5] |= q << (bit & 31);
-                    if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
+                    if constexpr (kBiasPack) {
+                        words[bit >> 5] += y << (bit & 31);
+                        if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] += (y & (uint32_t)qmax) >> (32 - (bit & 31));
+                    } else {
+                        const uint32_t q = y & (uint32_t)qmax;
+                        words[bit >> 5] |= q << (bit & 31);
+                        if ((bit & 31) + BITS > 32) words[(bit >> 5) + 1] |= q >> (32 - (bit & 31));
+                    }
                 };
                 uint32_t mk = 0;  // values within mu of a rounding boundary (bit k: column 32c + k)
                 if (fst && lm > 1.0f) {
@@ -789,8 +808,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                         t = fminf(fmaxf(t, 0.0f), qmaxf);
                         const float y = t + kMagic;
                         mk = __funnelshift_l(__float_as_uint(__fsub_rn(lm, fabsf(t - (y - kMagic)))), mk, 1);
-                        put(k, lv ? __float_as_uint(y) : 0u);
+                        put(k, lv ? __float_as_uint(y) : 0x4B400000u);  // dead block: q = 0
                     }
+                }
+                if constexpr (kBiasPack) {
+#pragma unroll
+                    for (int w = 0; w < BITS; w++) words[w] -= pack_bias<BITS>(w);
                 }
                 if (valid) {
                     uint32_t* dst = reinterpret_cast<uint32_t*>(crow) + c * BITS;
