@@ -57,7 +57,7 @@ constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
 constexpr int kThreads = 480;
 constexpr int kEpiWarp0 = 3;
-constexpr int kQCap = 24;             // repair jobs per warp and round
+constexpr int kQCap = 20;             // repair jobs per warp and round
 constexpr int kAcc = 4;               // accumulator buffers in tensor memory
 constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
@@ -68,7 +68,8 @@ struct EncSmem {
     static constexpr uint32_t stages = 0;
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
     static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 12 warps x kQCap x 8 B
-    static constexpr uint32_t misc = queue + 12 * kQCap * 8;
+    static constexpr uint32_t xch = queue + 12 * kQCap * 8;  // keys: 3 warpgroups x 2 x 4 warps x 4 floats
+    static constexpr uint32_t misc = xch + 3 * 2 * 4 * 4 * 4;
     static constexpr uint32_t total = misc + 384;  // base is 1024-aligned (checked in-kernel)
 };
 
@@ -81,6 +82,7 @@ struct Misc {
     int abort_flag;
     float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
     float gmaxb[kSegBufs][4];  // and max_i ||G_i||
+    uint64_t xbar[3][2];       // keys: per warpgroup, exchange of the group-norm maxima
 };
 
 static_assert(sizeof(Misc) <= 384, "Misc outgrew its shared-memory slot");
@@ -223,6 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
     unsigned char* stages = sm + EncSmem::stages;
     unsigned char* bsplit = sm + EncSmem::bsplit;
     uint32_t* queue = reinterpret_cast<uint32_t*>(sm + EncSmem::queue);
+    float* xch = reinterpret_cast<float*>(sm + EncSmem::xch);
 
     const RowArgs& a = P.a;
     const tc::Sched& S = P.S;
@@ -254,6 +257,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             mbar_init(&M->accempty[i], 4);
         }
         for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 1);
+        for (int w = 0; w < 3; w++) {
+            mbar_init(&M->xbar[w][0], 4);
+            mbar_init(&M->xbar[w][1], 4);
+        }
         mbar_init(&M->bfree, 1);
         M->abort_flag = 0;
         fence_barrier_init();
@@ -517,47 +524,58 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             float bs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
             if (KEYS) {
                 // a key block is one channel over the tile's 128 tokens: its bound uses the
-                // largest group norm among those tokens; each lane takes 4 token rows, then
-                // the warp reduces (every warp of the group computes it for itself)
-                float gm[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-#pragma unroll 1
-                for (int q = 0; q < 4; q++) {
-                    const int tr = lane + 32 * q;
-                    float gs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+                // largest group norm among those tokens. Each warp takes its own 32 token rows
+                // (one per lane); the four warps of the warpgroup then exchange their per-group
+                // maxima in shared memory (two buffers, alternating by tile)
+                float gs[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll 4
+                for (int c8 = 0; c8 < 16; c8++) {
+                    const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
+                                                                     (((c8 & 7) ^ (row & 7)) << 4));
+                    float s0 = bf_lo(xv.x) * bf_lo(xv.x);
+                    s0 = fmaf(bf_hi(xv.x), bf_hi(xv.x), s0);
+                    s0 = fmaf(bf_lo(xv.y), bf_lo(xv.y), s0);
+                    s0 = fmaf(bf_hi(xv.y), bf_hi(xv.y), s0);
+                    s0 = fmaf(bf_lo(xv.z), bf_lo(xv.z), s0);
+                    s0 = fmaf(bf_hi(xv.z), bf_hi(xv.z), s0);
+                    s0 = fmaf(bf_lo(xv.w), bf_lo(xv.w), s0);
+                    s0 = fmaf(bf_hi(xv.w), bf_hi(xv.w), s0);
+                    const int r = (c8 * 8) / g;  // g >= 32: at most 4 groups
+#pragma unroll
+                    for (int rr = 0; rr < 4; rr++)
+                        if (rr == r) gs[rr] += s0;
+                }
+                if (!(isfinite(gs[0]) && isfinite(gs[1]) && isfinite(gs[2]) && isfinite(gs[3]))) {
                     for (int c8 = 0; c8 < 16; c8++) {
-                        const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + tr * 128 +
-                                                                         (((c8 & 7) ^ (tr & 7)) << 4));
-                        float s0 = bf_lo(xv.x) * bf_lo(xv.x);
-                        s0 = fmaf(bf_hi(xv.x), bf_hi(xv.x), s0);
-                        s0 = fmaf(bf_lo(xv.y), bf_lo(xv.y), s0);
-                        s0 = fmaf(bf_hi(xv.y), bf_hi(xv.y), s0);
-                        s0 = fmaf(bf_lo(xv.z), bf_lo(xv.z), s0);
-                        s0 = fmaf(bf_hi(xv.z), bf_hi(xv.z), s0);
-                        s0 = fmaf(bf_lo(xv.w), bf_lo(xv.w), s0);
-                        s0 = fmaf(bf_hi(xv.w), bf_hi(xv.w), s0);
-                        const int r = (c8 * 8) / g;  // g >= 32: at most 4 groups
-#pragma unroll
-                        for (int rr = 0; rr < 4; rr++)
-                            if (rr == r) gs[rr] += s0;
-                    }
-#pragma unroll
-                    for (int rr = 0; rr < 4; rr++) gm[rr] = fmaxf(gm[rr], gs[rr]);
-                    if (!(isfinite(gs[0]) && isfinite(gs[1]) && isfinite(gs[2]) && isfinite(gs[3]))) {
-                        for (int c8 = 0; c8 < 16; c8++) {
-                            const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + tr * 128 +
-                                                                             (((c8 & 7) ^ (tr & 7)) << 4));
-                            const uint32_t wv[4] = {xv.x, xv.y, xv.z, xv.w};
-                            for (int k = 0; k < 4; k++)
-                                if (bf16_nonfinite(wv[k] & 0xffffu) || bf16_nonfinite(wv[k] >> 16))
-                                    flag |= CG_FLAG_NONFINITE_INPUT;
-                        }
+                        const uint4 xv = *reinterpret_cast<const uint4*>(stg + (c8 >> 3) * 16384 + row * 128 +
+                                                                         (((c8 & 7) ^ (row & 7)) << 4));
+                        const uint32_t wv[4] = {xv.x, xv.y, xv.z, xv.w};
+                        for (int k = 0; k < 4; k++)
+                            if (bf16_nonfinite(wv[k] & 0xffffu) || bf16_nonfinite(wv[k] >> 16))
+                                flag |= CG_FLAG_NONFINITE_INPUT;
                     }
                 }
 #pragma unroll
                 for (int rr = 0; rr < 4; rr++)
                     for (int off = 16; off >= 1; off >>= 1)
-                        gm[rr] = fmaxf(gm[rr], __shfl_xor_sync(0xffffffffu, gm[rr], off));
+                        gs[rr] = fmaxf(gs[rr], __shfl_xor_sync(0xffffffffu, gs[rr], off));
+                const int kx = (i - wg) / 3;  // this warpgroup's tile count
+                float* xb = xch + (wg * 2 + (kx & 1)) * 16;
+                if (lane == 0) {
+#pragma unroll
+                    for (int rr = 0; rr < 4; rr++) xb[q4 * 4 + rr] = gs[rr];
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&M->xbar[wg][kx & 1]);
+                const bool okx = mbar_wait(&M->xbar[wg][kx & 1], (kx >> 1) & 1, abort_flag, kWaitLimitNs);
+                if (!__all_sync(0xffffffffu, okx)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                float gm[4];
+#pragma unroll
+                for (int rr = 0; rr < 4; rr++)
+                    gm[rr] = fmaxf(fmaxf(xb[rr], xb[4 + rr]), fmaxf(xb[8 + rr], xb[12 + rr]));
                 bs[0] = pick4(gm, row / g);  // fmaxf keeps a NaN out; non-finite input is flagged above
             }
             // unroll depth measured per block count (code size against load parallelism)
