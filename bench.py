@@ -173,6 +173,19 @@ def cpu_sample(w, G, seconds=12.0, nthreads=None, start=0):
                       f"{t_total:.2f} s on {nthreads} threads"}
 
 
+def workload_config(w, ws):
+    """The `config` of a bench line for workload `w` on `ws` ranks (both arms print the same)."""
+    config = {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
+              "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
+              "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
+              "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
+              "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"}
+    if w.T_cap:
+        config.update({"T_cap": w.T_cap,
+                       "step": "append 1 token per sequence at T_cap - 1, decode all T_cap tokens"})
+    return config
+
+
 def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
@@ -195,7 +208,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": round(v, 4), "unit": "GB/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(el / args.steps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic", "config": {"workload": w.name},
+            "data": "synthetic", "config": workload_config(w, args.gpus),
             "cpu_baseline": {"value": round(v, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
                              "sample": vals[-1]["sample"]},
             "e2e": {"value": round(v, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -396,11 +409,7 @@ def run_cuda(args):
         raise RuntimeError(f"device status flags {flags} after the timed region")
 
     if rank == 0:
-        config = {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
-                  "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
-                  "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
-                  "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
-                  "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"}
+        config = workload_config(w, ws)
         config.update(P.config)
         line = {
             "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
