@@ -251,12 +251,44 @@ def _setup_cache(w, dev, ws, stream):
     hx = torch.from_numpy(x.reshape(-1).view(np.int16)).pin_memory()
     hout = torch.empty_like(hx).pin_memory()
 
-    def e2e_step():
+    # End to end, layers streamed through per-layer calls (the layout is layer-major, so a
+    # layer's input, codes, scales, residual and gauges are contiguous): the host->device copy
+    # of layer l+1 and the device->host copy of layer l-1 overlap the coding of layer l. Each
+    # step starts after the previous one has finished.
+    shape1 = cg.Shape(**{**w.shape, "L": 1})
+    nc1, ns1, nr1 = cg.packed_bytes(shape1, params)
+    px, pg = dx.numel() // w.L, dG.numel() // w.L
+    aligned = all(v % 16 == 0 for v in (nc1, ns1, nr1, 2 * px, 4 * pg))
+    s_in, s_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    ev_in = [torch.cuda.Event() for _ in range(w.L)]
+    ev_done = [torch.cuda.Event() for _ in range(w.L)]
+
+    def e2e_layers():
+        s_in.wait_stream(stream)
+        for l in range(w.L):
+            xs, gs = slice(l * px, (l + 1) * px), slice(l * pg, (l + 1) * pg)
+            with torch.cuda.stream(s_in):
+                dx[xs].copy_(hx[xs], non_blocking=True)
+                ev_in[l].record(s_in)
+            stream.wait_event(ev_in[l])
+            c1 = codes[l * nc1:(l + 1) * nc1]
+            sc1 = scales[l * (ns1 // 4):(l + 1) * (ns1 // 4)]
+            r1 = resid[l * (nr1 // 2):(l + 1) * (nr1 // 2)] if nr1 else None
+            cg.encode(shape1, params, dx[xs], dG[gs], c1, sc1, r1, stream=stream)
+            cg.decode(shape1, params, c1, sc1, r1, dG[gs], out[xs], stream=stream)
+            ev_done[l].record(stream)
+            s_out.wait_event(ev_done[l])
+            with torch.cuda.stream(s_out):
+                hout[xs].copy_(out[xs], non_blocking=True)
+        stream.wait_stream(s_out)
+
+    def e2e_whole():
         dx.copy_(hx, non_blocking=True)
         encode()
         decode()
         hout.copy_(out, non_blocking=True)
 
+    e2e_step = e2e_layers if (aligned and w.L > 1) else e2e_whole
     P.e2e_step, P.h2d, P.d2h = e2e_step, n, n
     P.e2e_bytes = 2 * n
     return P
