@@ -608,12 +608,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
 
-            // ---- 2. approximate block ranges from the accumulator, and per 32-column chunk the
-            // values within 2 Ep of the chunk's own min / max, Ep >= E (item 3) being known
-            // before the ranges are: any candidate extreme of a block is among them
+            // ---- 2. approximate block ranges from the accumulator. With two blocks per row the
+            // candidate masks are built here for every chunk (measured faster there): the values
+            // within 2 Ep of the chunk's own min / max, Ep >= E (item 3) being known before the
+            // ranges are. Otherwise they are built in the exact-extreme round, only where needed.
+            constexpr bool kEagerMasks = NBK == 2;
             float mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
             float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-            float clo[4], chi[4];           // chunk min / max
+            float clo[4], chi[4];           // chunk min / max (eager masks)
             uint32_t pm[4], px[4];          // chunk candidate masks (bit k = column 32c + k)
 #pragma unroll 1
             for (int c = 0; c < 4; c++) {
@@ -631,6 +633,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const int bk = (c * 32) / blk;
                 set4(mn, bk, fminf(pick4(mn, bk), lo));
                 set4(mx, bk, fmaxf(pick4(mx, bk), hi));
+                if constexpr (!kEagerMasks) continue;
                 // |z~| <= ||G_i|| ||x|| + E, so Ep bounds the E of item 3 from above
                 const float xn = sqrtf(pick4(bs, bk)) * 1.0001f;
                 const float ep = xn * M->emaxb[ls & 3][bk] + 2.0f * xn * M->gmaxb[ls & 3][bk] * 2.41e-7f;
@@ -674,17 +677,46 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
 
             // ---- 4. exact extremes of ambiguous blocks (warp-cooperative rounds)
             if (__any_sync(0xffffffffu, amb != 0)) {
-                // candidates: a chunk's values near its own min (max) are candidates of the
-                // block min (max) when the chunk min lies within 2E of the block min
+                if constexpr (kEagerMasks) {
+                    // candidates: a chunk's values near its own min (max) are candidates of the
+                    // block min (max) when the chunk min lies within 2E of the block min
 #pragma unroll 1
-                for (int c = 0; c < 4; c++) {
-                    const int bk = (c * 32) / blk;
-                    const int need = (amb >> (2 * bk)) & 3;
-                    const float e2 = 2.0f * pick4(E, bk);
-                    const bool nl = need && pick4(clo, c) <= __fadd_rn(pick4(mn, bk), e2);
-                    const bool nh = (need & 1) && pick4(chi, c) >= __fsub_rn(pick4(mx, bk), e2);
-                    set4(pm, c, nl ? pick4(pm, c) : 0u);
-                    set4(px, c, nh ? pick4(px, c) : 0u);
+                    for (int c = 0; c < 4; c++) {
+                        const int bk = (c * 32) / blk;
+                        const int need = (amb >> (2 * bk)) & 3;
+                        const float e2 = 2.0f * pick4(E, bk);
+                        const bool nl = need && pick4(clo, c) <= __fadd_rn(pick4(mn, bk), e2);
+                        const bool nh = (need & 1) && pick4(chi, c) >= __fsub_rn(pick4(mx, bk), e2);
+                        set4(pm, c, nl ? pick4(pm, c) : 0u);
+                        set4(px, c, nh ? pick4(px, c) : 0u);
+                    }
+                } else {
+                    // candidates of an ambiguous block's min (max): its values within 2E of the
+                    // approximate min (max); the chunks some lane needs are reloaded from TMEM
+#pragma unroll 1
+                    for (int c = 0; c < 4; c++) {
+                        const int bk = (c * 32) / blk;
+                        const int need = (amb >> (2 * bk)) & 3;
+                        uint32_t m0 = 0, m1 = 0;
+                        if (__any_sync(0xffffffffu, need != 0)) {
+                            uint32_t v[32];
+                            tmem_ld32(tacc + c * 32, v);
+                            tmem_wait_ld();
+                            const float e2 = 2.0f * pick4(E, bk);
+                            const float tl = __fadd_rn(pick4(mn, bk), e2), th = __fsub_rn(pick4(mx, bk), e2);
+                            uint32_t a0 = 0, a1 = 0;
+#pragma unroll
+                            for (int k = 31; k >= 0; k--) {
+                                const float z = __uint_as_float(v[k]);
+                                a0 = __funnelshift_l(__float_as_uint(__fsub_rn(tl, z)), a0, 1);
+                                a1 = __funnelshift_l(__float_as_uint(__fsub_rn(z, th)), a1, 1);
+                            }
+                            m0 = need ? ~a0 : 0u;        // z <= tl
+                            m1 = (need & 1) ? ~a1 : 0u;  // z >= th
+                        }
+                        set4(pm, c, m0);
+                        set4(px, c, m1);
+                    }
                 }
                 float ex_mn[4] = {INFINITY, INFINITY, INFINITY, INFINITY};
                 float ex_mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
