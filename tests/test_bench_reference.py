@@ -25,3 +25,21 @@ def test_reference_arm_line():
     import bench
     from paper_2607_20538_gb300 import synth
     assert line["config"] == bench.workload_config(synth.WORKLOADS["tiny"], 1)
+
+
+def test_reference_arm_two_ranks_prints_once():
+    """Launched as two ranks (torchrun, as the multi-GPU bench is), rank 0 alone runs and
+    prints; the other rank exits 0 without work."""
+    import socket
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        port = s.getsockname()[1]
+    r = subprocess.run([sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
+                        "--master-addr", "127.0.0.1", "--master-port", str(port), "bench.py", "--impl", "reference",
+                        "--workload", "tiny", "--steps", "2", "--warmup", "3", "--gpus", "2"],
+                       cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [l for l in r.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["n_gpus"] == 2
