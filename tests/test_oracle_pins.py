@@ -254,6 +254,47 @@ def test_identity_gauge_is_bare_backend(bits, blk, g):
             np.testing.assert_array_equal(oracle.unpack(codes[row, b], blk, bits), q)
 
 
+def _np_pack(q, bits):
+    """Little-endian bit stream of b-bit codes (bit 0 = LSB of byte 0), numpy only."""
+    bits_arr = ((np.asarray(q, np.uint32)[:, None] >> np.arange(bits, dtype=np.uint32)) & 1).astype(np.uint8)
+    return np.packbits(bits_arr.reshape(-1), bitorder="little")
+
+
+@pytest.mark.parametrize("bits,Gt,R", [(3, 32, 20), (4, 16, 0), (2, 32, 40)])
+def test_kivi_identity_gauge_is_bare_kivi(bits, Gt, R):
+    """Sec. 4.3 KIVI with the identity gauge: keys quantized per channel over groups of Gt
+    tokens, values per token over blocks of Gt channels, the newest T - n_q tokens kept raw.
+    The codes, scales and residual are rebuilt with numpy from the layouts alone (per-channel
+    key streams, then per-token value blocks) and the numpy block quantizer."""
+    w = _wl(L=1, B=2, H=2, T=150, d=32, group=8, backend=1, bits=bits, block=Gt, residual=R)
+    x = synth.kv_cache(w, threads=1)
+    r = oracle.encode(w.shape, w.params, x, synth.gauges(w, "identity"))
+    xf = _f32(x)
+    nq = max(0, (w.T - R) // Gt) * Gt
+    codes, scales = [], []
+    for b in range(w.B):          # keys [B][H][n_q/Gt][d]: one channel's Gt-token stream each
+        for h in range(w.H):
+            for grp in range(nq // Gt):
+                for c in range(w.d):
+                    s16, m16, q = _np_quantize(xf[0, 0, b, h, grp * Gt:(grp + 1) * Gt, c], bits)
+                    codes.append(_np_pack(q, bits))
+                    scales += [np.array(s16).view(np.uint16), np.array(m16).view(np.uint16)]
+    for b in range(w.B):          # values [B][H][n_q][d/Gt]: one token's Gt-channel block each
+        for h in range(w.H):
+            for t in range(nq):
+                for k in range(w.d // Gt):
+                    s16, m16, q = _np_quantize(xf[0, 1, b, h, t, k * Gt:(k + 1) * Gt], bits)
+                    codes.append(_np_pack(q, bits))
+                    scales += [np.array(s16).view(np.uint16), np.array(m16).view(np.uint16)]
+    want_codes = np.concatenate(codes) if codes else np.zeros(0, np.uint8)
+    np.testing.assert_array_equal(r["codes"][:want_codes.size], want_codes)
+    got_s = r["scales"][:len(scales)].view(np.float16).astype(np.float32)
+    want_s = np.array(scales, np.uint16).view(np.float16).astype(np.float32)
+    np.testing.assert_array_equal(got_s, want_s)
+    np.testing.assert_array_equal(r["residual"].reshape(w.L, 2, w.B, w.H, w.T - nq, w.d), x[..., nq:, :])
+    assert oracle.packed_bytes(w.shape, w.params) == (want_codes.size, 2 * len(scales), 2 * x[..., nq:, :].size)
+
+
 @pytest.mark.parametrize("bits,blk,g", [(4, 64, 128), (6, 32, 32), (3, 128, 64)])
 def test_block_ranges_brute_force_on_z(bits, blk, g):
     """Per-block min/max, scale, zero and codes recomputed by brute force from the
