@@ -11,6 +11,11 @@ e2e    = the same through the C ABI with host buffers: pinned host -> device cop
 roofline: the slower of the two kernels; algorithmic bytes per launch / its average
          CUDA-event duration, against the measured copy bandwidth.
 
+workloads: with the default 8B-shaped workload the same process then times the other target
+         workloads (27B-shaped 6-bit, KIVI-3, the rolling decode step) with fewer steps:
+         device-timed encode/decode ms, GB/s and HBM fractions per kernel.
+cpu_baseline: the oracle on the host cores (all of them, and one thread).
+
 Multi-GPU (torchrun): every rank encodes/decodes its own cache of the same shape (the
 units (l, s, b, h) are independent; no collective on the data path), weak scaling.
 --impl reference times the CPU oracle on the host cores on a bounded sample.
@@ -356,25 +361,12 @@ def _setup_rolling(w, dev, ws, stream):
     return P
 
 
-def run_cuda(args):
+def _time_problem(P, stream, steps: int, warmup: int, dev, ws: int, clock_dev: int):
+    """Warm-up, then `steps` timed steps of problem P on `stream` (CUDA events per kernel and
+    around the whole region, nvidia-smi clocks sampled during it)."""
     import torch
 
     import paper_2607_20538_gb300 as cg
-    from paper_2607_20538_gb300 import synth
-
-    ws, rank, local = _dist()
-    if ws > 1:
-        import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    else:
-        torch.cuda.set_device(0)
-    dev = torch.cuda.current_device()
-    w = synth.WORKLOADS[args.workload]
-    if args.layers:
-        w = w.replace(L=min(args.layers, w.L))
-    stream = torch.cuda.current_stream()
-    P = (_setup_rolling if w.T_cap else _setup_cache)(w, dev, ws, stream)
 
     def step(ev=None):
         if ev is not None:
@@ -386,14 +378,14 @@ def run_cuda(args):
         if ev is not None:
             ev[2].record(stream)
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         step()
     torch.cuda.synchronize()
     flags = cg.get_status()
     if flags:
         raise RuntimeError(f"device status flags {flags} after warm-up")
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
-    clocks = Clocks(dev if ws == 1 else local)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    clocks = Clocks(clock_dev)
     clocks.start()
     if ws > 1:
         torch.distributed.barrier()
@@ -401,20 +393,72 @@ def run_cuda(args):
     t_start = torch.cuda.Event(enable_timing=True)
     t_end = torch.cuda.Event(enable_timing=True)
     t_start.record(stream)
-    for i in range(args.steps):
+    for i in range(steps):
         step(evs[i])
     t_end.record(stream)
     torch.cuda.synchronize()
     if ws > 1:
         torch.distributed.barrier()
     clk = clocks.stop()
-    total_ms = t_start.elapsed_time(t_end)
-    enc_ms = [e[0].elapsed_time(e[1]) for e in evs]
-    dec_ms = [e[1].elapsed_time(e[2]) for e in evs]
-    total_ms = rank_reduce(total_ms, "max", dev)
-    ms_step = total_ms / args.steps
+    flags = cg.get_status()
+    if flags:
+        raise RuntimeError(f"device status flags {flags} after the timed region")
+    total_ms = rank_reduce(t_start.elapsed_time(t_end), "max", dev)
+    return {"ms_step": total_ms / steps,
+            "enc_ms": statistics.mean(e[0].elapsed_time(e[1]) for e in evs),
+            "dec_ms": statistics.mean(e[1].elapsed_time(e[2]) for e in evs),
+            "clocks": clk}
+
+
+def _kernel_figures(P, t, peak):
+    return {"encode_ms": round(t["enc_ms"], 5), "decode_ms": round(t["dec_ms"], 5),
+            "encode_gbs": round(P.enc_bytes / (t["enc_ms"] * 1e-3) / 1e9, 2),
+            "decode_gbs": round(P.dec_bytes / (t["dec_ms"] * 1e-3) / 1e9, 2),
+            "enc_frac": round(P.enc_alg / (t["enc_ms"] * 1e-3) / 1e9 / peak, 4),
+            "dec_frac": round(P.dec_alg / (t["dec_ms"] * 1e-3) / 1e9 / peak, 4),
+            "enc_alg_bytes": P.enc_alg, "dec_alg_bytes": P.dec_alg}
+
+
+# Context only: the paper prints no encode/decode throughput; these are its own figures for
+# the storage/timing side of the method and the hardware it states.
+PAPER_CONTEXT = {
+    "hardware": "NVIDIA RTX PRO 6000 Blackwell (CC 12.0, 97,887 MiB), AMD Ryzen 9 9950X, CUDA 13.2, PyTorch 2.12.1",
+    "throughput": "not reported (the serial storage/timing run is shown as a normalized figure only)",
+    "zfp4_actual_bits_per_value": 4.0,
+    "zfp_rate_accuracy_bits_per_value": 6e-5,
+    "inverse_gauge_round_trip_nrmse": "< 5.1e-8 (identity clone: 0)",
+    "kl_reduction_learned_gauge": {"block_uniform": "44.2% (18/18 pairs)", "kivi": "27.2% (18/18 pairs)"},
+}
+
+# The other target workloads, timed in the same process after the headline one.
+EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling")
+
+
+def run_cuda(args):
+    import gc
+
+    import torch
+
+    from paper_2607_20538_gb300 import synth
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+    clock_dev = dev if ws == 1 else local
+    w = synth.WORKLOADS[args.workload]
+    if args.layers:
+        w = w.replace(L=min(args.layers, w.L))
+    stream = torch.cuda.current_stream()
+    P = (_setup_rolling if w.T_cap else _setup_cache)(w, dev, ws, stream)
+    t = _time_problem(P, stream, args.steps, args.warmup, dev, ws, clock_dev)
+    ms_step = t["ms_step"]
     value = job_throughput(P.enc_bytes + P.dec_bytes, ws, ms_step)
-    enc_avg, dec_avg = statistics.mean(enc_ms), statistics.mean(dec_ms)
+    enc_avg, dec_avg = t["enc_ms"], t["dec_ms"]
     peak, peak_kind = _peaks()
     if dec_avg >= enc_avg:
         dom, dom_ms, dom_alg = "decode", dec_avg, P.dec_alg
@@ -436,10 +480,12 @@ def run_cuda(args):
     torch.cuda.synchronize()
     e2e_ms = rank_reduce(e0.elapsed_time(e1) / e2e_steps, "max", dev)
     e2e_val = job_throughput(P.e2e_bytes, ws, e2e_ms)
+    import paper_2607_20538_gb300 as cg
     flags = cg.get_status()
     if flags:
-        raise RuntimeError(f"device status flags {flags} after the timed region")
+        raise RuntimeError(f"device status flags {flags} after the end-to-end steps")
 
+    line = None
     if rank == 0:
         config = workload_config(w, ws)
         config.update(P.config)
@@ -460,10 +506,43 @@ def run_cuda(args):
             "e2e": {"value": round(e2e_val, 2), "unit": "GB/s", "h2d_bytes_per_step": P.h2d,
                     "d2h_bytes_per_step": P.d2h},
             "gpu_launches": P.launches * args.steps,
-            "clocks": clk,
+            "clocks": t["clocks"],
+            "paper_context": PAPER_CONTEXT,
         }
+    G_main = P.G
+    del P
+    gc.collect()
+    torch.cuda.empty_cache()
+
+    # the other target workloads, device-timed in the same process (fewer steps)
+    extra = {}
+    if not args.layers and not args.no_extra and args.workload == "llama3_8b":
+        for name in EXTRA_WORKLOADS:
+            we = synth.WORKLOADS[name]
+            Pe = (_setup_rolling if we.T_cap else _setup_cache)(we, dev, ws, stream)
+            te = _time_problem(Pe, stream, args.extra_steps, 3, dev, ws, clock_dev)
+            fig = _kernel_figures(Pe, te, peak)
+            fig["steps"] = args.extra_steps
+            fig["ms_per_step"] = round(te["ms_step"], 5)
+            fig["value_gbs"] = round(job_throughput(Pe.enc_bytes + Pe.dec_bytes, ws, te["ms_step"]), 2)
+            if we.T_cap:
+                fig["steps_per_s"] = round(1e3 / te["ms_step"], 3)
+            fig["config"] = {**workload_config(we, ws), **Pe.config}
+            fig["gpu_launches_per_step"] = Pe.launches
+            fig["clocks"] = te["clocks"]
+            extra[name] = fig
+            del Pe
+            gc.collect()
+            torch.cuda.empty_cache()
+
+    if rank == 0:
+        if extra:
+            line["workloads"] = extra
         if not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_sample(w, P.G, seconds=args.cpu_seconds)
+            line["cpu_baseline"] = cpu_sample(w, G_main, seconds=args.cpu_seconds)
+            one = cpu_sample(w, G_main, seconds=args.cpu_seconds_1t, nthreads=1)
+            line["cpu_baseline"]["one_thread"] = {"value": one["value"], "unit": one["unit"], "cores": 1,
+                                                  "sample": one["sample"]}
         print(json.dumps(line), flush=True)
     if ws > 1:
         torch.distributed.destroy_process_group()
@@ -479,7 +558,11 @@ def main():
     ap.add_argument("--layers", type=int, default=0,
                     help="keep only the first N layers of the workload (small cases for profiling)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-seconds-1t", type=float, default=4.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="time only --workload (by default the 8B-shaped headline run also times the other targets)")
+    ap.add_argument("--extra-steps", type=int, default=10)
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

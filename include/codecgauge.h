@@ -17,8 +17,11 @@
  *   - All data pointers are DEVICE pointers owned by the caller. The library never
  *     allocates, frees or retains them. Calls are asynchronous on `stream`
  *     (a cudaStream_t passed as void*; NULL = legacy default stream).
- *   - Every entry point returns an int status: CG_OK or a negative CG_E* code. On a
- *     negative status nothing was launched; cg_last_error() returns a message.
+ *   - Every entry point returns an int status: CG_OK or a negative CG_E* code. On
+ *     CG_EINVAL, CG_EUNSUPPORTED and CG_ERANGE nothing was launched. A KIVI call launches
+ *     up to three kernels (keys, values, residual copy) in order, so a CG_ECUDA from it may
+ *     follow launches that were already queued; the outputs are then invalid.
+ *     cg_last_error() returns a message.
  *   - Numbers: bf16 = IEEE binary16-brain (8-bit significand), fp16 = IEEE binary16,
  *     fp32 = IEEE binary32, all little-endian.
  *
@@ -127,8 +130,15 @@ int cg_decode(const cg_shape* shape, const cg_params* params,
               const void* codes, const void* scales, const void* residual,
               const float* gauges, void* out_kv_bf16, void* stream);
 
-/* Synchronizes `stream`, returns the accumulated CG_FLAG_* bits of the current device in
- * *device_flags and clears them. Returns CG_ECUDA if the synchronize fails. */
+/* Reads and clears (in one atomic step, ordered on `stream`) the accumulated CG_FLAG_* bits
+ * of the current device, synchronizes `stream` and returns them in *device_flags. Returns
+ * CG_ECUDA if a launch, copy or the synchronize fails. The limit of each bounded pipeline
+ * wait in the tensor-core kernels is 4 s; the environment variable CODECGAUGE_PIPE_WAIT_NS
+ * (read at every encode/decode call, nanoseconds, at most 4e9; other values are ignored)
+ * lowers it. It is a diagnostic knob: below 1 ms the waits poll without suspending, so a
+ * limit of a few hundred nanoseconds makes them give up and raise CG_FLAG_PIPE_TIMEOUT
+ * without any fault (the outputs of that call are then invalid). The drains of copies
+ * already in flight keep the 4 s limit. */
 int cg_get_status(void* stream, int32_t* device_flags);
 
 /* Message for the most recent failing call on this host thread ("" if none). The pointer

@@ -7,8 +7,11 @@
 #include <mutex>
 #include <string>
 
+#include <cstdlib>
+
 #include "cg_launch.h"
 #include "cg_tc.h"
+#include "cg_tc_common.cuh"
 
 // The library is built with hidden symbol visibility; only the C ABI is exported.
 #define CG_EXPORT __attribute__((visibility("default")))
@@ -16,6 +19,11 @@
 namespace cg {
 
 __device__ int32_t g_status_word = 0;
+__device__ int32_t g_status_taken = 0;
+
+// Reads and clears the status word in one atomic step, on the caller's stream, so a flag
+// raised by a kernel on another stream between a read and a clear cannot be lost.
+__global__ void status_take_kernel(int32_t* status, int32_t* taken) { *taken = atomicExch(status, 0); }
 
 namespace {
 
@@ -193,8 +201,21 @@ void kivi_value_maps(const cg_shape* sh, const Sizes& z, RowMap* cm, RowMap* sm)
     sm->base = BH * z.key_scales_per_bh;
 }
 
+// Limit of each bounded pipeline wait in the tensor-core kernels: 4 s, or the value of the
+// environment variable CODECGAUGE_PIPE_WAIT_NS (a diagnostic knob: a tiny limit makes the
+// waits give up, which exercises the CG_FLAG_PIPE_TIMEOUT path without any fault). The
+// drains of copies already issued always keep the 4 s limit.
+uint64_t pipe_wait_ns() {
+    const char* v = getenv("CODECGAUGE_PIPE_WAIT_NS");
+    if (!v || !*v) return tc::kWaitLimitNs;
+    char* end = nullptr;
+    const unsigned long long n = strtoull(v, &end, 10);
+    return (end && *end == 0 && n <= tc::kWaitLimitNs) ? (uint64_t)n : tc::kWaitLimitNs;
+}
+
 RowArgs row_args(const cg_shape* sh, const cg_params* p, int32_t* status) {
     RowArgs a{};
+    a.wait_ns = pipe_wait_ns();
     a.status = status;
     a.L = sh->L;
     a.B = sh->B;
@@ -403,15 +424,18 @@ CG_EXPORT int cg_get_status(void* stream, int32_t* device_flags) {
     int32_t* status = nullptr;
     int rc = status_ptr(&status);
     if (rc) return rc;
+    int32_t* taken = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void**>(&taken), g_status_taken);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status slot)");
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    cudaError_t e = cudaStreamSynchronize(st);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+    status_take_kernel<<<1, 1, 0, st>>>(status, taken);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "status read launch");
     int32_t v = 0;
-    e = cudaMemcpy(&v, status, sizeof v, cudaMemcpyDeviceToHost);
+    e = cudaMemcpyAsync(&v, taken, sizeof v, cudaMemcpyDeviceToHost, st);
     if (e != cudaSuccess) return cuda_fail(e, "read status");
-    const int32_t zero = 0;
-    e = cudaMemcpy(status, &zero, sizeof zero, cudaMemcpyHostToDevice);
-    if (e != cudaSuccess) return cuda_fail(e, "clear status");
+    e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
     *device_flags = v;
     return CG_OK;
 }

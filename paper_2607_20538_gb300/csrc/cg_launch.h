@@ -23,6 +23,7 @@ struct RowArgs {
     int64_t T_x;            // tokens per unit in the dense x / out tensor
     int64_t t_count;        // tokens processed per unit
     int none_mode;          // 1 = CG_NONE (codes hold fp32 z rows)
+    uint64_t wait_ns;       // limit of each bounded pipeline wait of the tensor-core kernels
     RowMap cmap;            // byte offset of a row's codes
     RowMap smap;            // u32 index of a row's first block scale
 };

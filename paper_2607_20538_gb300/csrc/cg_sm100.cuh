@@ -49,12 +49,36 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+__device__ __forceinline__ bool mbar_test_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait on an mbarrier phase. Gives up after `limit_ns` of wall time, or as soon as
 // *abort becomes non-zero (another warp gave up); returns false in both cases.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const volatile int* abort,
-                                          uint64_t limit_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
+// try_wait may suspend the thread for a while before it reports an incomplete phase; with
+// the default limit (seconds) the clock and the abort flag are read every 64 attempts,
+// which keeps the spin light. A limit below 1 ms is a diagnostic setting: the wait then
+// polls with the non-suspending test_wait and reads the clock after every attempt, so that
+// a limit of well under a microsecond runs out before any pipeline stage can complete.
+// Everything after the first attempt is out of line, which keeps the kernels' code small.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, const volatile int* abort,
+                                                   uint64_t limit_ns) {
     const uint64_t t0 = globaltimer_ns();
+    if (limit_ns < 1000000ull) {
+        for (;;) {
+            if (mbar_test_wait(bar, parity)) return true;
+            if (*abort) return false;
+            if (globaltimer_ns() - t0 > limit_ns) return false;
+        }
+    }
     for (uint32_t it = 0;; it++) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((it & 63u) == 63u) {
@@ -62,6 +86,12 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
             if (globaltimer_ns() - t0 > limit_ns) return false;
         }
     }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const volatile int* abort,
+                                          uint64_t limit_ns) {
+    if (limit_ns >= 1000000ull && mbar_try_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, abort, limit_ns);
 }
 
 // ---------------------------------------------------------------- TMA

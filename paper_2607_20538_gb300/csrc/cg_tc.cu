@@ -287,7 +287,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             it.init(a, S, t_begin);
             for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
                 const int st = i % kStages;
-                if (!mbar_wait(&M->empty[st], ((i / kStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                if (!mbar_wait(&M->empty[st], ((i / kStages) & 1) ^ 1, abort_flag, a.wait_ns)) {
                     *abort_flag = 1;
                     break;
                 }
@@ -320,12 +320,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 const int64_t ls = ti.seg - seg0;
                 bool ok = true;
                 if (ti.seg != cur) {
-                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, a.wait_ns);
                     cur = ti.seg;
                 }
                 const int st = i % kStages, buf = i % kAcc;
-                ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
-                ok = ok && mbar_wait(&M->accempty[buf], ((i / kAcc) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, a.wait_ns);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i / kAcc) & 1) ^ 1, abort_flag, a.wait_ns);
                 if (!ok) {
                     *abort_flag = 1;
                     break;
@@ -379,7 +379,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             if (ti.seg == cur) continue;
             const int64_t ls = ti.seg - seg0;
             if (nconv > 0) {
-                const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, a.wait_ns);
                 if (!__all_sync(0xffffffffu, ok)) {
                     *abort_flag = 1;
                     break;
@@ -507,9 +507,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
             const int st = i % kStages, buf = i % kAcc;
-            bool ok = mbar_wait(&M->accfull[buf], (i / kAcc) & 1, abort_flag, kWaitLimitNs);
-            ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, kWaitLimitNs);
-            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+            bool ok = mbar_wait(&M->accfull[buf], (i / kAcc) & 1, abort_flag, a.wait_ns);
+            ok = ok && mbar_wait(&M->full[st], (i / kStages) & 1, abort_flag, a.wait_ns);
+            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
                 break;
@@ -567,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&M->xbar[wg][kx & 1]);
-                const bool okx = mbar_wait(&M->xbar[wg][kx & 1], (kx >> 1) & 1, abort_flag, kWaitLimitNs);
+                const bool okx = mbar_wait(&M->xbar[wg][kx & 1], (kx >> 1) & 1, abort_flag, a.wait_ns);
                 if (!__all_sync(0xffffffffu, okx)) {
                     *abort_flag = 1;
                     break;

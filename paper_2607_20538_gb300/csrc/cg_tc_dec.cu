@@ -4,7 +4,8 @@
 // Persistent warp-specialized kernel, one CTA per SM, 14 warps:
 //   warp 0      bulk-copy producer: the packed codes of a 128-token tile are contiguous
 //               (rows of 16*bits bytes); one cp.async.bulk per tile into a ring of stages;
-//   warp 1      MMA issuer: D_k = A_k B^T on tcgen05, A = codes as bf16 (128 + q, exact),
+//   warp 1      MMA issuer: D_k = A_k B^T on tcgen05, A = codes as bf16 (2^b + q, exact;
+//               8-bit codes as q),
 //               B = G^T of the gauge group split into two bf16 terms; one fp32
 //               accumulator per quantization sub-block k of a group (block < group gives
 //               two), double buffered in tensor memory (tile i uses buffer i mod 2);
@@ -13,15 +14,19 @@
 //               sum_{j in sub-block k} G[j][i] of the split;
 //   warps 6..13 epilogue: both warpgroups work on every tile, warpgroup h on output
 //               columns 64h..64h+63, one token row (TMEM lane) per thread:
-//               xhat_i = sum_k s_k * D_k[i] + (m_k - 128 s_k) * c_k[i]. The accumulator
+//               xhat_i = sum_k s_k * D_k[i] + (m_k - 2^b s_k) * c_k[i]. The accumulator
 //               buffer is released as soon as it is in registers, so the MMAs of tile i+2
 //               overlap the arithmetic of tile i; each warp stages its 32 x 64 bf16 block
 //               in shared memory (128-byte swizzle) and writes it with one TMA tile store.
 //               Each thread loads the next tile's block scales one tile ahead.
 // With the scale and zero of a block constant along the token, dequantization commutes
-// with the rotation, so the integer codes go through the tensor cores unscaled. The number
-// of sub-block accumulators is a template parameter, so each kernel holds only its own
-// epilogue.
+// with the rotation, so the integer codes go through the tensor cores unscaled. In real
+// arithmetic s_k D_k + (m_k - 2^b s_k) c_k = sum_j (hi + lo)_ji zhat_j, so the split residual
+// of G is not amplified by the offset; the offset only scales the fp32 rounding of D_k and of
+// the zero-point term, which is why it is the smallest power of two that keeps 2^b + q a
+// plain bit pattern (2^b + q has b significant bits below its leading one), and why c_k is
+// a compensated sum. The number of sub-block accumulators is a template parameter, so each
+// kernel holds only its own epilogue.
 #include <cuda_bf16.h>
 
 #include "cg_sm100.cuh"
@@ -78,20 +83,29 @@ struct DecParams {
     int nsub;  // accumulators per gauge group: group / block when block < group, else 1
 };
 
-// codes of one row (128 codes, little-endian bit stream) -> 16 chunks of 8 bf16 (128 + q)
+// bf16 bit pattern of 2^BITS + q (q < 2^BITS): exponent of 2^BITS, q in the top BITS of the
+// 7 mantissa bits
+template <int BITS>
+__host__ __device__ constexpr uint32_t code_bf16_base() {
+    return (uint32_t)(127 + BITS) << 7;
+}
+
+// codes of one row (128 codes, little-endian bit stream) -> 16 chunks of 8 bf16 (2^b + q; 8-bit
+// codes as q)
 template <int BITS>
 __device__ __forceinline__ void unpack_row(const uint32_t* w, uint4 (&out)[16]) {
     if constexpr (BITS == 4) {
-        // eight nibbles per word: split low/high nibbles, interleave them back into code
-        // order with byte permutes, then pair each code byte with the 0x43 exponent byte
+        // eight nibbles per word: place the low/high nibbles at mantissa bits 3..6 of their
+        // bytes (with the exponent's low bit 0x80), interleave them back into code order
+        // with byte permutes, then pair each byte with the 0x41 exponent byte (16 + q)
 #pragma unroll
         for (int c = 0; c < 16; c++) {
-            const uint32_t lo_n = w[c] & 0x0F0F0F0Fu;         // codes 0, 2, 4, 6 of the word
-            const uint32_t hi_n = (w[c] >> 4) & 0x0F0F0F0Fu;  // codes 1, 3, 5, 7
+            const uint32_t lo_n = ((w[c] << 3) & 0x78787878u) | 0x80808080u;  // codes 0, 2, 4, 6
+            const uint32_t hi_n = ((w[c] >> 1) & 0x78787878u) | 0x80808080u;  // codes 1, 3, 5, 7
             const uint32_t q03 = __byte_perm(lo_n, hi_n, 0x5140);  // codes 0..3 as bytes
             const uint32_t q47 = __byte_perm(lo_n, hi_n, 0x7362);  // codes 4..7
-            out[c] = make_uint4(__byte_perm(q03, 0x43u, 0x4140), __byte_perm(q03, 0x43u, 0x4342),
-                                __byte_perm(q47, 0x43u, 0x4140), __byte_perm(q47, 0x43u, 0x4342));
+            out[c] = make_uint4(__byte_perm(q03, 0x41u, 0x4140), __byte_perm(q03, 0x41u, 0x4342),
+                                __byte_perm(q47, 0x41u, 0x4140), __byte_perm(q47, 0x41u, 0x4342));
         }
     } else {
 #pragma unroll
@@ -109,7 +123,8 @@ __device__ __forceinline__ void unpack_row(const uint32_t* w, uint4 (&out)[16]) 
                     q[h] = v & ((1u << BITS) - 1u);
                 }
                 if (BITS < 8) {
-                    o[e] = 0x43004300u | q[0] | (q[1] << 16);
+                    constexpr uint32_t base = code_bf16_base<BITS>() * 0x10001u;
+                    o[e] = base | (q[0] << (7 - BITS)) | (q[1] << (23 - BITS));
                 } else {
                     const __nv_bfloat162 b2 = __floats2bfloat162_rn((float)q[0], (float)q[1]);
                     o[e] = *reinterpret_cast<const uint32_t*>(&b2);
@@ -143,7 +158,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
     const uint32_t bsz = (g == 128) ? 32768u : 16384u;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     constexpr int kRowBytes = 16 * BITS;
-    constexpr float kOff = BITS < 8 ? 128.0f : 0.0f;
+    constexpr float kOff = BITS < 8 ? (float)(1 << BITS) : 0.0f;
 
     const int64_t t_begin = S.n_tiles * blockIdx.x / gridDim.x;
     const int64_t t_end = S.n_tiles * (blockIdx.x + 1) / gridDim.x;
@@ -188,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
             it.init(a, S, t_begin);
             for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
                 const int st = i % kCStages;
-                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, a.wait_ns)) {
                     *abort_flag = 1;
                     break;
                 }
@@ -250,12 +265,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 const int64_t ls = ti.seg - seg0;
                 bool ok = true;
                 if (ti.seg != cur) {
-                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, a.wait_ns);
                     cur = ti.seg;
                 }
                 const int ab = i & 1, buf = i & 1;
-                ok = ok && mbar_wait(&M->afull[ab], (i >> 1) & 1, abort_flag, kWaitLimitNs);
-                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->afull[ab], (i >> 1) & 1, abort_flag, a.wait_ns);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, a.wait_ns);
                 if (!ok) {
                     *abort_flag = 1;
                     break;
@@ -292,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 const int64_t ls = ti.seg - seg0;
                 if (nconv > 0) {
                     // the MMAs of the previous gauge set must be done with B
-                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, a.wait_ns);
                     if (!__all_sync(0xffffffffu, ok)) {
                         *abort_flag = 1;
                         break;
@@ -301,7 +316,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 // B[n][k] = G_r[k - r g][n - r g]: thread `row` builds output channel n = row
                 const int n = row, r = n / g, i_in = n - r * g;
                 const float* Gc = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g + (int64_t)r * g * g + i_in;
-                float cs0 = 0.0f, cs1 = 0.0f;
+                // c_k: the split's (hi + lo) values summed by a pairwise tree over each step's
+                // eight, the step sums accumulated with compensation (Neumaier), so c_k is within
+                // a few u of its value (fp64 arithmetic is far slower on this part)
+                float cs0 = 0.0f, ce0 = 0.0f, cs1 = 0.0f, ce1 = 0.0f;
+                auto kadd = [](float& sum, float& comp, float v) {
+                    const float t = sum + v;
+                    comp += fabsf(sum) >= fabsf(v) ? (sum - t) + v : (v - t) + sum;
+                    sum = t;
+                };
+                float tv[8];
                 for (int j = 0; j < g; j += 8) {
                     uint32_t hi[4], lo[4];
 #pragma unroll
@@ -313,11 +337,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                         const __nv_bfloat16 l1 = __float2bfloat16_rn(v1 - __bfloat162float(h1));
                         hi[e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
                         lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
-                        const float t2 = (__bfloat162float(h0) + __bfloat162float(l0)) +
-                                         (__bfloat162float(h1) + __bfloat162float(l1));
-                        if (nsub > 1 && j + e >= blk) cs1 += t2;
-                        else cs0 += t2;
+                        tv[e] = __bfloat162float(h0) + __bfloat162float(l0);  // exact
+                        tv[e + 1] = __bfloat162float(h1) + __bfloat162float(l1);
                     }
+                    const float t8 = ((tv[0] + tv[1]) + (tv[2] + tv[3])) + ((tv[4] + tv[5]) + (tv[6] + tv[7]));
+                    // blk is a multiple of 8, so the eight values of a step share a sub-block
+                    if (nsub > 1 && j >= blk) kadd(cs1, ce1, t8);
+                    else kadd(cs0, ce0, t8);
                     const int k = r * g + j;
                     unsigned char* reg1 = bsplit + 1 * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
                     unsigned char* reg0 = bsplit + 0 * bsz + (g == 128 ? (k >> 6) * 16384 : 0);
@@ -325,8 +351,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                     *reinterpret_cast<uint4*>(reg0 + sw128_offset(n, k & 63)) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
                 }
                 float* cb = csum + (ls & 3) * 2 * kD;
-                cb[n] = cs0;
-                cb[kD + n] = cs1;
+                cb[n] = cs0 + ce0;
+                cb[kD + n] = cs1 + ce1;
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
@@ -334,8 +360,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 nconv++;
             }
             const int st = i % kCStages, ab = i & 1;
-            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, kWaitLimitNs);
-            ok = ok && mbar_wait(&M->aempty[ab], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, a.wait_ns);
+            ok = ok && mbar_wait(&M->aempty[ab], ((i >> 1) & 1) ^ 1, abort_flag, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
                 break;
@@ -397,8 +423,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                 nx.step(a, 1);
                 load_scales(nx.info(a), sz_next);
             }
-            bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
-            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+            bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, a.wait_ns);
+            ok = ok && mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
                 break;

@@ -137,7 +137,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
             it.init(a, S, t_begin);
             for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
                 const int st = i % kCStages;
-                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, kWaitLimitNs)) {
+                if (!mbar_wait(&M->cempty[st], ((i / kCStages) & 1) ^ 1, abort_flag, a.wait_ns)) {
                     *abort_flag = 1;
                     break;
                 }
@@ -185,12 +185,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 const int64_t ls = ti.seg - seg0;
                 bool ok = true;
                 if (ti.seg != cur) {
-                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, kWaitLimitNs);
+                    ok = mbar_wait(&M->gready[ls & 3], (ls >> 2) & 1, abort_flag, a.wait_ns);
                     cur = ti.seg;
                 }
                 const int ab = i % kAStages, buf = i & 1;
-                ok = ok && mbar_wait(&M->afull[ab], (i / kAStages) & 1, abort_flag, kWaitLimitNs);
-                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, kWaitLimitNs);
+                ok = ok && mbar_wait(&M->afull[ab], (i / kAStages) & 1, abort_flag, a.wait_ns);
+                ok = ok && mbar_wait(&M->accempty[buf], ((i >> 1) & 1) ^ 1, abort_flag, a.wait_ns);
                 if (!ok) {
                     *abort_flag = 1;
                     break;
@@ -226,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
             if (ti.seg != cur && half == 0) {
                 const int64_t ls = ti.seg - seg0;
                 if (nconv > 0) {
-                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, kWaitLimitNs);
+                    const bool ok = mbar_wait(&M->bfree, (nconv - 1) & 1, abort_flag, a.wait_ns);
                     if (!__all_sync(0xffffffffu, ok)) {
                         *abort_flag = 1;
                         break;
@@ -259,8 +259,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 nconv++;
             }
             const int st = i % kCStages, ab = i % kAStages;
-            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, kWaitLimitNs);
-            ok = ok && mbar_wait(&M->aempty[ab], ((i / kAStages) & 1) ^ 1, abort_flag, kWaitLimitNs);
+            bool ok = mbar_wait(&M->cfull[st], (i / kCStages) & 1, abort_flag, a.wait_ns);
+            ok = ok && mbar_wait(&M->aempty[ab], ((i / kAStages) & 1) ^ 1, abort_flag, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
                 break;
@@ -322,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
         for (int i = 0; i < my_tiles; i++, it.step(a, 1)) {
             const tc::TileInfo ti = it.info(a);
             const int buf = i & 1;
-            const bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, kWaitLimitNs);
+            const bool ok = mbar_wait(&M->accfull[buf], (i >> 1) & 1, abort_flag, a.wait_ns);
             if (!__all_sync(0xffffffffu, ok)) {
                 *abort_flag = 1;
                 break;

@@ -53,7 +53,10 @@ def _check_unit(w, G, x_unit, l, h, codes_u8, scales_u16, resid_u16, out_u16):
         np.testing.assert_array_equal(resid_u16, ref["residual"])
     xr = oracle.decode(w1.shape, w1.params, ref["codes"], ref["scales"], ref["residual"], G1)
     step = scales_as_elements(w1, ref["scales"]) * mism if mism.any() else None
-    compare_decode(w1, out_u16, xr, G1, step)
+    st = compare_decode(w1, out_u16, xr, G1, step, codes=ref["codes"], scales_u16=ref["scales"])
+    print(f"unit (l={l}, h={h}): {int(mism.sum())} flagged code mismatches of {mism.size}; decode checked "
+          f"tightly on {st['tight']} values ({st['tight_not_rne']} not bf16(ref)); "
+          f"{st['rms_floor_only']} pass only through the rms floor")
 
 
 @pytest.fixture(autouse=True)

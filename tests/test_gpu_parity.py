@@ -104,13 +104,15 @@ def test_encode_decode_parity(name):
         np.testing.assert_array_equal(_host_u16(resid, nr), ref["residual"])
     # end to end: GPU decode of the GPU's own buffers
     got = gpu_decode(w, codes, scales, resid, dG)
-    compare_decode(w, got, xr, G, step_mism)
+    packed = {} if w.backend == 2 else dict(codes=ref["codes"], scales_u16=ref["scales"])
+    compare_decode(w, got, xr, G, step_mism, **packed)
     # identical packed input: GPU decode of the oracle's bytes, no flag allowance
     oc = torch.from_numpy(np.concatenate([ref["codes"], np.zeros(16, np.uint8)])).cuda()
     os_ = torch.from_numpy(np.concatenate([ref["scales"], np.zeros(8, np.uint16)]).view(np.int16)).cuda()
     orr = torch.from_numpy(np.concatenate([ref["residual"], np.zeros(8, np.uint16)]).view(np.int16)).cuda()
     got2 = gpu_decode(w, oc, os_, orr, dG)
-    compare_decode(w, got2, xr, G, None)
+    st = compare_decode(w, got2, xr, G, None, **packed)
+    assert st["tight"] == (xr.size if packed else 0)
     assert cg.get_status() == 0
 
 
@@ -174,7 +176,7 @@ def test_rolling_append_and_window_decode():
     cg.decode(win, params, codes, scales, None, dG, out)
     xr = oracle.decode(w.shape, w.params, ref["codes"], ref["scales"], ref["residual"], G)
     step = scales_as_elements(w, ref["scales"]) * mism if mism.any() else None
-    compare_decode(w, out.cpu().numpy().view(np.uint16), xr, G, step)
+    compare_decode(w, out.cpu().numpy().view(np.uint16), xr, G, step, codes=ref["codes"], scales_u16=ref["scales"])
     # a window in the middle of the history: tokens [5, 17)
     mid = cg.Shape(L=w.L, B=w.B, H=w.H, T=12, d=w.d, t0=5, T_cap=Tc)
     out2 = torch.empty(w.L * 2 * w.B * w.H * 12 * w.d, dtype=torch.int16, device="cuda")

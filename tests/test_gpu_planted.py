@@ -99,4 +99,4 @@ def test_planted_kivi_keys_and_values():
     cg.decode(shape, params, codes, scales, resid, dG, out)
     xr = oracle.decode(w.shape, w.params, ref["codes"], ref["scales"], ref["residual"], G)
     step = scales_as_elements(w, ref["scales"]) * mism if mism.any() else None
-    compare_decode(w, out.cpu().numpy().view(np.uint16), xr, G, step)
+    compare_decode(w, out.cpu().numpy().view(np.uint16), xr, G, step, codes=ref["codes"], scales_u16=ref["scales"])
