@@ -962,16 +962,12 @@ cudaError_t launch_encode_nbk(const EncParams& P, const CUtensorMap& map, cudaSt
     return cudaGetLastError();
 }
 
-// keys: one block (the 128-token group) per channel; rows: 128 / block blocks per row
+// keys: one block (the 128-token group) per channel (block-uniform and KIVI value rows are
+// encoded by cg_tc_rows.cu)
 template <int BITS, bool KEYS>
 cudaError_t launch_encode_bits(const EncParams& P, const CUtensorMap& map, cudaStream_t st) {
-    if constexpr (KEYS) {
-        return launch_encode_nbk<BITS, KEYS, 1>(P, map, st);
-    } else {
-        if (P.a.blk == 128) return launch_encode_nbk<BITS, KEYS, 1>(P, map, st);
-        if (P.a.blk == 64) return launch_encode_nbk<BITS, KEYS, 2>(P, map, st);
-        return launch_encode_nbk<BITS, KEYS, 4>(P, map, st);
-    }
+    static_assert(KEYS, "rows are encoded by tc_rows_encode_kernel");
+    return launch_encode_nbk<BITS, KEYS, 1>(P, map, st);
 }
 
 template <bool KEYS>
@@ -994,18 +990,6 @@ cudaError_t launch_encode(const RowArgs& a, cudaStream_t st) {
 }
 
 }  // namespace
-
-bool tc_row_encode_eligible(const RowArgs& a) {
-    if (a.d != kD || a.none_mode) return false;
-    if (!(a.blk == 32 || a.blk == 64 || a.blk == 128)) return false;
-    if (a.t_count < 64) return false;
-    const int64_t rows = (int64_t)a.L * 2 * a.B * a.H * a.T_x;
-    if (rows + 128 >= (int64_t)1 << 31) return false;
-    if ((reinterpret_cast<uintptr_t>(a.x) & 15u) || (reinterpret_cast<uintptr_t>(a.codes) & 15u)) return false;
-    return tmap_encode_fn() != nullptr;
-}
-
-cudaError_t tc_launch_row_encode(const RowArgs& a, cudaStream_t st) { return launch_encode<false>(a, st); }
 
 // KIVI keys as rows of the key tensor: s = 0 only, block = the 128-token key group, t_count
 // = the quantized tokens (whole groups); cmap/smap address a group's first token (the
