@@ -44,6 +44,7 @@
 #include "cg_sm100.cuh"
 #include "cg_tc.h"
 #include "cg_tc_common.cuh"
+#include "cg_tc_enc.cuh"
 #include "cg_tmap.h"
 
 namespace cg {
@@ -61,7 +62,6 @@ constexpr int kQCap = 20;             // repair jobs per warp and round
 constexpr int kAcc = 4;               // accumulator buffers in tensor memory
 constexpr int kNPass = 3;             // bf16 terms of the gauge split
 constexpr int kSegBufs = 4;
-constexpr float kU = 5.9604645e-08f;  // 2^-24
 constexpr float kMagic = 12582912.0f; // 1.5 * 2^23: adding it rounds to an integer (RNE)
 
 struct EncSmem {
@@ -363,13 +363,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
         }
     } else if (warp == 2) {
         // ------------------------------------------------------------ gauge converter
-        const int lg = 31 - __clz(g);
-        const float c_order = (float)(1 + lg) * kU * 1.01f;
-        // the split's two small terms are accumulated first (their partial sums stay below
-        // 2^-8 of the group's scale), so the accumulation error is dominated by the n_hi
-        // K-steps of the leading term; 4 u covers the rounding inside each MMA and of the result
-        const int n_hi = (KEYS ? 128 : gb) / 16;
-        const float c_tc = ((float)n_hi + 4.0f + (float)((npass - 1) * n_hi) * (1.0f / 128.0f)) * kU;
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
@@ -386,97 +379,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_encode_kernel(const __grid_con
                 }
             }
             const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
-            {
-                // warm L2 with the next gauge set of this CTA (read at the next conversion)
-                int nl = ti.l, ns = ti.s, nh = ti.h + 1;
-                if (nh == a.H) {
-                    nh = 0;
-                    if (++ns == a.s_lo + a.s_n) {
-                        ns = a.s_lo;
-                        nl++;
-                    }
-                }
-                if (nl < a.L) {
-                    const char* nG = reinterpret_cast<const char*>(a.G + ((int64_t)(nl * 2 + ns) * a.H + nh) * (int64_t)kD * g);
-                    for (int off = lane * 128; off < kD * g * 4; off += 32 * 128)
-                        asm volatile("prefetch.global.L2 [%0];" ::"l"(nG + off));
-                }
-            }
-            float e_row[4], s_g2[4], s_res2[4];
-#pragma unroll
-            for (int q = 0; q < 4; q++) s_g2[q] = s_res2[q] = 0.0f;
-            for (int j = 0; j < g; j += 8) {
-                // the four rows of this lane: eight loads in flight per step
-                float4 v0[4], v1[4];
-#pragma unroll
-                for (int q = 0; q < 4; q++) {
-                    const float* Gr = Gf + (size_t)(lane + 32 * q) * g;
-                    v0[q] = __ldg(reinterpret_cast<const float4*>(Gr + j));
-                    v1[q] = __ldg(reinterpret_cast<const float4*>(Gr + j + 4));
-                }
-#pragma unroll
-                for (int q = 0; q < 4; q++) {
-                    const int n = lane + 32 * q;  // B row = output channel
-                    const int k = (n / g) * g + j;
-                    const float v[8] = {v0[q].x, v0[q].y, v0[q].z, v0[q].w, v1[q].x, v1[q].y, v1[q].z, v1[q].w};
-                    uint32_t term[3][4];
-#pragma unroll
-                    for (int e = 0; e < 8; e += 2) {
-                        float rest0 = v[e], rest1 = v[e + 1];
-                        s_g2[q] = fmaf(v[e], v[e], s_g2[q]);
-                        s_g2[q] = fmaf(v[e + 1], v[e + 1], s_g2[q]);
-#pragma unroll
-                        for (int t = 0; t < 3; t++) {
-                            const __nv_bfloat16 h0 = __float2bfloat16_rn(rest0);
-                            const __nv_bfloat16 h1 = __float2bfloat16_rn(rest1);
-                            rest0 = __fsub_rn(rest0, __bfloat162float(h0));
-                            rest1 = __fsub_rn(rest1, __bfloat162float(h1));
-                            term[t][e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) |
-                                              ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-                        }
-                        s_res2[q] = fmaf(rest0, rest0, s_res2[q]);
-                        s_res2[q] = fmaf(rest1, rest1, s_res2[q]);
-                    }
-#pragma unroll
-                    for (int t = 0; t < 3; t++) {
-                        unsigned char* region = bsplit + (npass - 1 - t) * bsz + (fullk ? (k >> 6) * 16384 : 0);
-                        *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
-                            make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
-                    }
-                }
-            }
-#pragma unroll
-            for (int q = 0; q < 4; q++)
-                e_row[q] = ((c_order + c_tc) * sqrtf(s_g2[q]) + sqrtf(s_res2[q])) * 1.001f + 1e-30f;
-            // per quantization block: max of e over the rows that bound its values (keys: a
-            // block is one channel over tokens, bounded by the max over all rows, slot 0)
-#pragma unroll
-            for (int bk = 0; bk < 4; bk++) {
-                if (KEYS ? bk == 0 : bk < nbk) {
-                    int lo = 0, hi = 128;
-                    if (!KEYS) bound_range(bk, g, blk, lo, hi);
-                    float m = 0.0f;
-#pragma unroll
-                    for (int q = 0; q < 4; q++) {
-                        const int n = lane + 32 * q;
-                        if (n >= lo && n < hi) m = fmaxf(m, e_row[q]);
-                    }
-                    float gm = 0.0f;  // max_i ||G_i|| over the same rows: bounds |z~| / ||x||
-#pragma unroll
-                    for (int q = 0; q < 4; q++) {
-                        const int n = lane + 32 * q;
-                        if (n >= lo && n < hi) gm = fmaxf(gm, sqrtf(s_g2[q]));
-                    }
-                    for (int off = 16; off >= 1; off >>= 1) {
-                        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
-                        gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, off));
-                    }
-                    if (lane == 0) {
-                        M->emaxb[ls & 3][bk] = m;
-                        M->gmaxb[ls & 3][bk] = gm;
-                    }
-                }
-            }
+            tce::prefetch_next_gauges(a, ti, g, lane);
+            tce::convert_gauge_set<KEYS, 4>(Gf, g, blk, nbk, fullk, bsz, bsplit, M->emaxb[ls & 3], M->gmaxb[ls & 3], 0, lane);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&M->gready[ls & 3]);

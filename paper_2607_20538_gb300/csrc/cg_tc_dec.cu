@@ -326,19 +326,31 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                     sum = t;
                 };
                 float tv[8];
+                // eight gauge values per step; the next step's loads are in flight while this
+                // step converts (a gauge change stalls the MMAs until it is done)
+                float nv[8];
+#pragma unroll
+                for (int e = 0; e < 8; e++) nv[e] = __ldg(Gc + (int64_t)e * g);
                 for (int j = 0; j < g; j += 8) {
+                    float cv[8];
+#pragma unroll
+                    for (int e = 0; e < 8; e++) cv[e] = nv[e];
+                    if (j + 8 < g) {
+#pragma unroll
+                        for (int e = 0; e < 8; e++) nv[e] = __ldg(Gc + (int64_t)(j + 8 + e) * g);
+                    }
                     uint32_t hi[4], lo[4];
 #pragma unroll
                     for (int e = 0; e < 8; e += 2) {
-                        const float v0 = __ldg(Gc + (int64_t)(j + e) * g);
-                        const float v1 = __ldg(Gc + (int64_t)(j + e + 1) * g);
-                        const __nv_bfloat16 h0 = __float2bfloat16_rn(v0), h1 = __float2bfloat16_rn(v1);
-                        const __nv_bfloat16 l0 = __float2bfloat16_rn(v0 - __bfloat162float(h0));
-                        const __nv_bfloat16 l1 = __float2bfloat16_rn(v1 - __bfloat162float(h1));
-                        hi[e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-                        lo[e >> 1] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
-                        tv[e] = __bfloat162float(h0) + __bfloat162float(l0);  // exact
-                        tv[e + 1] = __bfloat162float(h1) + __bfloat162float(l1);
+                        // both values to bf16 in one conversion (round to nearest even)
+                        const __nv_bfloat162 h = __float22bfloat162_rn(make_float2(cv[e], cv[e + 1]));
+                        const float2 hf = __bfloat1622float2(h);
+                        const __nv_bfloat162 l = __float22bfloat162_rn(make_float2(cv[e] - hf.x, cv[e + 1] - hf.y));
+                        const float2 lf = __bfloat1622float2(l);
+                        hi[e >> 1] = *reinterpret_cast<const uint32_t*>(&h);
+                        lo[e >> 1] = *reinterpret_cast<const uint32_t*>(&l);
+                        tv[e] = hf.x + lf.x;  // exact
+                        tv[e + 1] = hf.y + lf.y;
                     }
                     const float t8 = ((tv[0] + tv[1]) + (tv[2] + tv[3])) + ((tv[4] + tv[5]) + (tv[6] + tv[7]));
                     // blk is a multiple of 8, so the eight values of a step share a sub-block

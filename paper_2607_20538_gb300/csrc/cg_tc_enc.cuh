@@ -9,7 +9,7 @@
 //     e_i = (c_order + c_tc) ||G_i||_2 + ||G_i - sum of split terms||_2,
 // c_order = (1 + log2 g) u the rounding bound of the fixed order, c_tc a bound on the
 // tensor-core fp32 accumulation: the MMAs accumulate the split's two small terms first
-// (partial sums below 2^-8 of ||G_i|| ||x||, 2 n_hi K-steps) and the leading term last
+// (partial sums below 2^-7 of ||G_i|| ||x||, 2 n_hi K-steps) and the leading term last
 // (n_hi = K / 16 steps), so c_tc = (n_hi + 4 + 2 n_hi / 128) u, 4 u covering the rounding
 // inside each MMA and of the result; the measured |z~ - Gx| stays below 2.4 u ||G_i|| ||x||
 // (g = 32 and 128; random, Hadamard and DCT gauges). Candidates that the bound leaves
@@ -152,65 +152,79 @@ __device__ __forceinline__ void prefetch_next_gauges(const RowArgs& a, const tc:
     }
 }
 
-// One warp converts the gauge set Gf (d/g diagonal g x g blocks, fp32) into the MMA's B
-// operand: output channel n = lane + 32 q is B row n, its K entries the gauge row; the three
-// bf16 terms of the exact split go to bsplit + (npass - 1 - t) * bsz (the smallest term is
-// accumulated first). Layout: full K = 128 (`fullk`, block-diagonal for g < 128) in two
-// 64-column SW128 halves of 16 KB, or one g-wide K block per group in a 64-column tile.
+// Converts rows of the gauge set Gf (d/g diagonal g x g blocks, fp32) into the MMA's B
+// operand: output channel n is B row n, its K entries the gauge row. A lane takes the NQ
+// rows n = lane + 32 q, q0 <= q < q0 + NQ, so one to four warps can share a set. The split
+// is exact by truncation: hi = v with its low 16 bits cleared, lo the same of v - hi, lo2
+// of the rest (for normal values nothing remains; a remainder is bounded below); the terms
+// go to bsplit + (npass - 1 - t) * bsz, so the smallest is accumulated first (|lo| < 2^-7
+// |hi|, |lo2| < 2^-14 |hi|). Layout: full K = 128 (`fullk`, block-diagonal for g < 128) in
+// two 64-column SW128 halves of 16 KB, or one g-wide K block per group in a 64-column tile.
 // Writes, per quantization block bk < nbk (keys: slot 0 for all rows), the largest bound
-// coefficient e_i over the rows that bound the block (emax[bk]) and the largest ||G_i||
-// (gmax[bk]).
-template <bool KEYS>
+// coefficient e_i over this warp's rows that bound the block (emax[bk]) and the largest
+// ||G_i|| among them (gmax[bk]); the readers take the maximum over the warps.
+template <bool KEYS, int NQ>
 __device__ __forceinline__ void convert_gauge_set(const float* Gf, int g, int blk, int nbk, bool fullk, uint32_t bsz,
-                                                  unsigned char* bsplit, float* emax, float* gmax, int lane) {
+                                                  unsigned char* bsplit, float* emax, float* gmax, int q0, int lane) {
     const int lg = 31 - __clz(g);
     const float c_order = (float)(1 + lg) * kU * 1.01f;
     const int n_hi = (KEYS ? 128 : (g < 16 ? 16 : g)) / 16;
     const float c_tc = ((float)n_hi + 4.0f + (float)((kNPass - 1) * n_hi) * (1.0f / 128.0f)) * kU;
-    float e_row[4], s_g2[4], s_res2[4];
+    float e_row[NQ], s_g2[NQ], s_res2[NQ];
 #pragma unroll
-    for (int q = 0; q < 4; q++) s_g2[q] = s_res2[q] = 0.0f;
+    for (int q = 0; q < NQ; q++) s_g2[q] = s_res2[q] = 0.0f;
+    // eight values of each row per step; the next step's loads are in flight while this step
+    // converts (a gauge change stalls the MMAs until the set is ready)
+    float4 n0[NQ], n1[NQ];
+#pragma unroll
+    for (int q = 0; q < NQ; q++) {
+        const float* Gr = Gf + (size_t)(lane + 32 * (q0 + q)) * g;
+        n0[q] = __ldg(reinterpret_cast<const float4*>(Gr));
+        n1[q] = __ldg(reinterpret_cast<const float4*>(Gr + 4));
+    }
     for (int j = 0; j < g; j += 8) {
-        // the four rows of this lane: eight loads in flight per step
-        float4 v0[4], v1[4];
+        float4 v0[NQ], v1[NQ];
 #pragma unroll
-        for (int q = 0; q < 4; q++) {
-            const float* Gr = Gf + (size_t)(lane + 32 * q) * g;
-            v0[q] = __ldg(reinterpret_cast<const float4*>(Gr + j));
-            v1[q] = __ldg(reinterpret_cast<const float4*>(Gr + j + 4));
+        for (int q = 0; q < NQ; q++) {
+            v0[q] = n0[q];
+            v1[q] = n1[q];
+        }
+        if (j + 8 < g) {
+#pragma unroll
+            for (int q = 0; q < NQ; q++) {
+                const float* Gr = Gf + (size_t)(lane + 32 * (q0 + q)) * g;
+                n0[q] = __ldg(reinterpret_cast<const float4*>(Gr + j + 8));
+                n1[q] = __ldg(reinterpret_cast<const float4*>(Gr + j + 12));
+            }
         }
 #pragma unroll
-        for (int q = 0; q < 4; q++) {
-            const int n = lane + 32 * q;  // B row = output channel
+        for (int q = 0; q < NQ; q++) {
+            const int n = lane + 32 * (q0 + q);  // B row = output channel
             const int k = (n / g) * g + j;
             const float v[8] = {v0[q].x, v0[q].y, v0[q].z, v0[q].w, v1[q].x, v1[q].y, v1[q].z, v1[q].w};
-            uint32_t term[3][4];
+            uint32_t tb[3][8];  // term bit patterns (fp32 with the low 16 bits clear)
 #pragma unroll
-            for (int e = 0; e < 8; e += 2) {
-                float rest0 = v[e], rest1 = v[e + 1];
+            for (int e = 0; e < 8; e++) {
+                float rest = v[e];
                 s_g2[q] = fmaf(v[e], v[e], s_g2[q]);
-                s_g2[q] = fmaf(v[e + 1], v[e + 1], s_g2[q]);
 #pragma unroll
                 for (int t = 0; t < 3; t++) {
-                    const __nv_bfloat16 h0 = __float2bfloat16_rn(rest0);
-                    const __nv_bfloat16 h1 = __float2bfloat16_rn(rest1);
-                    rest0 = __fsub_rn(rest0, __bfloat162float(h0));
-                    rest1 = __fsub_rn(rest1, __bfloat162float(h1));
-                    term[t][e >> 1] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+                    tb[t][e] = __float_as_uint(rest) & 0xffff0000u;
+                    rest = __fsub_rn(rest, __uint_as_float(tb[t][e]));  // exact
                 }
-                s_res2[q] = fmaf(rest0, rest0, s_res2[q]);
-                s_res2[q] = fmaf(rest1, rest1, s_res2[q]);
+                s_res2[q] = fmaf(rest, rest, s_res2[q]);
             }
 #pragma unroll
             for (int t = 0; t < 3; t++) {
                 unsigned char* region = bsplit + (kNPass - 1 - t) * bsz + (fullk ? (k >> 6) * 16384 : 0);
                 *reinterpret_cast<uint4*>(region + sw128_offset(n, k & 63)) =
-                    make_uint4(term[t][0], term[t][1], term[t][2], term[t][3]);
+                    make_uint4(__byte_perm(tb[t][0], tb[t][1], 0x7632), __byte_perm(tb[t][2], tb[t][3], 0x7632),
+                               __byte_perm(tb[t][4], tb[t][5], 0x7632), __byte_perm(tb[t][6], tb[t][7], 0x7632));
             }
         }
     }
 #pragma unroll
-    for (int q = 0; q < 4; q++) e_row[q] = ((c_order + c_tc) * sqrtf(s_g2[q]) + sqrtf(s_res2[q])) * 1.001f + 1e-30f;
+    for (int q = 0; q < NQ; q++) e_row[q] = ((c_order + c_tc) * sqrtf(s_g2[q]) + sqrtf(s_res2[q])) * 1.001f + 1e-30f;
     // per quantization block: max of e over the rows that bound its values (keys: a block is
     // one channel over tokens, bounded by the max over all rows, slot 0)
 #pragma unroll
@@ -220,8 +234,8 @@ __device__ __forceinline__ void convert_gauge_set(const float* Gf, int g, int bl
             if (!KEYS) bound_range(bk, g, blk, lo, hi);
             float m = 0.0f, gm = 0.0f;  // gm: max_i ||G_i|| over the same rows, bounds |z~| / ||x||
 #pragma unroll
-            for (int q = 0; q < 4; q++) {
-                const int n = lane + 32 * q;
+            for (int q = 0; q < NQ; q++) {
+                const int n = lane + 32 * (q0 + q);
                 if (n >= lo && n < hi) {
                     m = fmaxf(m, e_row[q]);
                     gm = fmaxf(gm, sqrtf(s_g2[q]));

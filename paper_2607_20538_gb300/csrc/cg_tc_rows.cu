@@ -2,14 +2,15 @@
 // rotation (Sec. 3, Z = G X) fused with the block-uniform quantizer of Sec. 4.3 (one range
 // per block of `block` channels of a token), also used for KIVI value rows.
 //
-// Persistent warp-specialized kernel, one CTA per SM, 15 warps:
+// Persistent warp-specialized kernel, one CTA per SM, 16 warps:
 //   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte
 //               swizzle) into a 4-stage ring;
 //   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group, one
 //               MMA chain per group block), G split into three bf16 terms (cg_tc_enc.cuh);
 //               fp32 accumulators in tensor memory, four buffers;
-//   warp 2      gauge converter: at each gauge change builds the split operand and the
-//               per-block error coefficients of the new gauge set;
+//   warps 2, 15 gauge converters: at each gauge change they build the split operand and
+//               the per-block error coefficients of the new gauge set (half of its rows each;
+//               the MMAs wait for it, so it is kept short);
 //   warps 3..14 three epilogue warpgroups; warpgroup k takes tiles i = k (mod 3); one
 //               thread per token row (= TMEM lane).
 //
@@ -32,8 +33,9 @@
 //      every lane's block needs no clamp and no boundary check (the usual case), else the
 //      checked loop, which clamps and marks values within mu of a rounding boundary;
 //   6. marked values (only when mu >= 1e-4, e.g. 8-bit codes) are recomputed and patched.
-// The block index of every 32-column chunk is a compile-time constant (the block count is
-// a template parameter), so the per-block state lives in registers without selects.
+// The block count is a template parameter, so the per-block state of a row takes only the
+// registers it needs; the chunk loops are not unrolled (the epilogue's code size sets its
+// instruction-fetch stalls) and pick a chunk's block values with selects.
 #include "cg_tc.h"
 #include "cg_tc_enc.cuh"
 #include "cg_tmap.h"
@@ -47,7 +49,8 @@ using tc::kWaitLimitNs;
 
 constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
-constexpr int kThreads = 480;
+constexpr int kThreads = 512;
+constexpr int kConvWarp1 = 15;  // second gauge-converter warp (the first is warp 2)
 constexpr int kEpiWarp0 = 3;
 constexpr int kQCap = 20;  // repair jobs per warp and round
 constexpr int kAcc = 4;    // accumulator buffers in tensor memory
@@ -57,7 +60,7 @@ struct RowSmem {
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
     static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 12 warps x kQCap x 8 B
     static constexpr uint32_t misc = queue + 12 * kQCap * 8;
-    static constexpr uint32_t total = misc + 384;  // base is 1024-aligned (checked in-kernel)
+    static constexpr uint32_t total = misc + 512;  // base is 1024-aligned (checked in-kernel)
 };
 
 struct RowMisc {
@@ -67,11 +70,11 @@ struct RowMisc {
     uint64_t bfree;
     uint32_t tmem_slot;
     int abort_flag;
-    float emaxb[kSegBufs][4];  // per gauge set and quantization block: max_i e_i
-    float gmaxb[kSegBufs][4];  // and max_i ||G_i||
+    float emaxb[kSegBufs][2][4];  // per gauge set, converter warp and quantization block: max_i e_i
+    float gmaxb[kSegBufs][2][4];  // and max_i ||G_i||
 };
 
-static_assert(sizeof(RowMisc) <= 384, "RowMisc outgrew its shared-memory slot");
+static_assert(sizeof(RowMisc) <= 512, "RowMisc outgrew its shared-memory slot");
 static_assert(RowSmem::total <= 232448, "row encode kernel exceeds 227 KB of shared memory");
 
 struct RowEncParams {
@@ -207,7 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
             mbar_init(&M->accfull[i], 1);
             mbar_init(&M->accempty[i], 4);
         }
-        for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 1);
+        for (int i = 0; i < kSegBufs; i++) mbar_init(&M->gready[i], 2);
         mbar_init(&M->bfree, 1);
         M->abort_flag = 0;
         fence_barrier_init();
@@ -255,8 +258,26 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
+        // A tile is always 24 MMAs (3 split terms x 128 / 16 K-steps, in one chain per gauge
+        // group). Their B descriptors, A offsets and accumulator columns are laid out once,
+        // so per tile the single issuing thread only adds the stage's A base: descriptor
+        // arithmetic in that thread would otherwise set the pace of the whole pipeline.
         if (lane == 0 && my_tiles > 0) {
+            constexpr int kMma = kNPass * (kD / 16);
             const uint32_t idesc = idesc_bf16_f32(128, gb);
+            uint64_t bdesc[kMma];
+            uint32_t aoff[kMma], doff[kMma], accb = 0;
+#pragma unroll
+            for (int q = 0; q < kMma; q++) {
+                const int p = q / (kD / 16), kk = q % (kD / 16);  // pass, K-step over the row
+                const int r = (kk * 16) / gb, ks = kk - r * (gb / 16);
+                const int k0 = kk * 16;
+                aoff[q] = (uint32_t)(((k0 >> 6) * 16384 + (k0 & 63) * 2) >> 4);
+                bdesc[q] = sdesc_sw128(smem_u32(bsplit) + p * bsz + (fullk ? (k0 >> 6) * 16384 : 0) + (r * gb) * 128 +
+                                       (k0 & 63) * 2);
+                doff[q] = (uint32_t)(r * gb);
+                accb |= (uint32_t)(p > 0 || ks > 0) << q;
+            }
             int64_t cur = -1;
             int committed = 0;
             tc::TileIter it;
@@ -277,21 +298,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                     break;
                 }
                 tc_fence_after();
-                const uint32_t a_base = smem_u32(stages + st * kTileBytes);
+                const uint64_t adesc = sdesc_sw128(smem_u32(stages + st * kTileBytes));
                 const uint32_t d_base = tmem + buf * 128;
-                for (int p = 0; p < kNPass; p++) {
-                    const uint32_t b_base = smem_u32(bsplit) + p * bsz;
-                    for (int r = 0; r < 128 / gb; r++) {
-                        for (int ks = 0; ks < gb / 16; ks++) {
-                            const int k0 = r * gb + ks * 16;
-                            const uint32_t a_addr = a_base + (k0 >> 6) * 16384 + (k0 & 63) * 2;
-                            const uint32_t b_addr = b_base + (fullk ? (k0 >> 6) * 16384 : 0) + (r * gb) * 128 + (k0 & 63) * 2;
-                            // D[token][channel] = x G^T, one chain per gauge group
-                            mma_bf16(d_base + r * gb, sdesc_sw128(a_addr), sdesc_sw128(b_addr), idesc,
-                                     (p > 0 || ks > 0) ? 1u : 0u);
-                        }
-                    }
-                }
+                // D[token][channel] = x G^T, one chain per gauge group
+#pragma unroll
+                for (int q = 0; q < kMma; q++) mma_bf16(d_base + doff[q], adesc + aoff[q], bdesc[q], idesc, (accb >> q) & 1u);
                 mma_commit(&M->accfull[buf]);
                 const bool last_of_seg = (i + 1 == my_tiles) || it.seg_last(a);
                 if (last_of_seg) mma_commit(&M->bfree);
@@ -303,8 +314,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                 mbar_wait(&M->accfull[i % kAcc], (i / kAcc) & 1, &zero, kWaitLimitNs);
             }
         }
-    } else if (warp == 2) {
-        // ------------------------------------------------------------ gauge converter
+    } else if (warp == 2 || warp == kConvWarp1) {
+        // ------------------------------------------------------------ gauge converters
+        // (two warps, 64 of the 128 gauge rows each)
+        const int cw = warp == 2 ? 0 : 1;
         int64_t cur = -1;
         int nconv = 0;
         tc::TileIter it;
@@ -321,8 +334,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                 }
             }
             const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
-            prefetch_next_gauges(a, ti, g, lane);
-            convert_gauge_set<false>(Gf, g, blk, NBK, fullk, bsz, bsplit, M->emaxb[ls & 3], M->gmaxb[ls & 3], lane);
+            if (cw == 0) prefetch_next_gauges(a, ti, g, lane);
+            convert_gauge_set<false, 2>(Gf, g, blk, NBK, fullk, bsz, bsplit, M->emaxb[ls & 3][cw], M->gmaxb[ls & 3][cw],
+                                        2 * cw, lane);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
@@ -421,7 +435,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
             int amb = 0;  // bit 2bk: scale needs the exact extremes; bit 2bk+1: zero needs the exact min
 #pragma unroll
             for (int bk = 0; bk < NBK; bk++) {
-                E[bk] = sqrtf(nb[bk]) * 1.0001f * M->emaxb[ls & 3][bk] + (fabsf(mn[bk]) + fabsf(mx[bk])) * 2.4e-7f;
+                const float emax = fmaxf(M->emaxb[ls & 3][0][bk], M->emaxb[ls & 3][1][bk]);
+                E[bk] = sqrtf(nb[bk]) * 1.0001f * emax + (fabsf(mn[bk]) + fabsf(mx[bk])) * 2.4e-7f;
                 const float e = E[bk];
                 const float mn_lo = __fsub_rn(mn[bk], e), mn_hi = __fadd_rn(mn[bk], e);
                 const float mx_lo = __fsub_rn(mx[bk], e), mx_hi = __fadd_rn(mx[bk], e);
