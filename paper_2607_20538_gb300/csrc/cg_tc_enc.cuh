@@ -67,7 +67,7 @@ __host__ __device__ __forceinline__ void bound_range(int bk, int g, int blk, int
 // staged bf16 tile (two 64-column halves, 128-byte swizzle), Gf the gauge set in global
 // memory.
 template <int kSlots>
-__device__ __noinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned char* stage, const float* Gf, int g,
+__device__ __forceinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned char* stage, const float* Gf, int g,
                                       int lane) {
     const int lgT = 29 - __clz(g);  // log2(g / 4); g in {8, ..., 128}
     const int T = 1 << lgT, teams = 32 >> lgT;
@@ -162,9 +162,10 @@ __device__ __forceinline__ void prefetch_next_gauges(const RowArgs& a, const tc:
 // two 64-column SW128 halves of 16 KB, or one g-wide K block per group in a 64-column tile.
 // Writes, per quantization block bk < nbk (keys: slot 0 for all rows), the largest bound
 // coefficient e_i over this warp's rows that bound the block (emax[bk]) and the largest
-// ||G_i|| among them (gmax[bk]); the readers take the maximum over the warps.
+// ||G_i|| among them (gmax[bk]); the readers take the maximum over the warps. Returns true
+// when the split of every row of this warp is exact (no remainder: normal values).
 template <bool KEYS, int NQ>
-__device__ __forceinline__ void convert_gauge_set(const float* Gf, int g, int blk, int nbk, bool fullk, uint32_t bsz,
+__device__ __forceinline__ bool convert_gauge_set(const float* Gf, int g, int blk, int nbk, bool fullk, uint32_t bsz,
                                                   unsigned char* bsplit, float* emax, float* gmax, int q0, int lane) {
     const int lg = 31 - __clz(g);
     const float c_order = (float)(1 + lg) * kU * 1.01f;
@@ -251,6 +252,10 @@ __device__ __forceinline__ void convert_gauge_set(const float* Gf, int g, int bl
             }
         }
     }
+    bool rem = false;
+#pragma unroll
+    for (int q = 0; q < NQ; q++) rem = rem || s_res2[q] != 0.0f;
+    return !__any_sync(0xffffffffu, rem);
 }
 
 }  // namespace tce

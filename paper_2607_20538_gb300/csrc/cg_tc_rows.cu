@@ -2,17 +2,18 @@
 // rotation (Sec. 3, Z = G X) fused with the block-uniform quantizer of Sec. 4.3 (one range
 // per block of `block` channels of a token), also used for KIVI value rows.
 //
-// Persistent warp-specialized kernel, one CTA per SM, 16 warps:
+// Persistent warp-specialized kernel, one CTA per SM, 20 warps:
 //   warp 0      TMA producer: 128-token x tiles (2 x [128 rows x 64 bf16], 128-byte
 //               swizzle) into a 4-stage ring;
 //   warp 1      MMA issuer: z~ = x G^T on tcgen05 (M = 128 tokens, N = K = gauge group, one
 //               MMA chain per group block), G split into three bf16 terms (cg_tc_enc.cuh);
 //               fp32 accumulators in tensor memory, four buffers;
-//   warps 2, 15 gauge converters: at each gauge change they build the split operand and
+//   warps 2, 19 gauge converters: at each gauge change they build the split operand and
 //               the per-block error coefficients of the new gauge set (half of its rows each;
 //               the MMAs wait for it, so it is kept short);
-//   warps 3..14 three epilogue warpgroups; warpgroup k takes tiles i = k (mod 3); one
-//               thread per token row (= TMEM lane).
+//   warps 3..18 four epilogue warpgroups; warpgroup k takes tiles i = k (mod 4); one
+//               thread per token row (= TMEM lane). Four warps per SMSP hide more of the
+//               epilogue's latencies than three; the kernel fits in 96 registers a thread.
 //
 // Epilogue of a tile, per row:
 //   1. the group norms ||x_R||_2 that scale the error bound, from the staged tile with
@@ -49,8 +50,9 @@ using tc::kWaitLimitNs;
 
 constexpr int kStages = 4;
 constexpr int kTileBytes = 128 * kD * 2;
-constexpr int kThreads = 512;
-constexpr int kConvWarp1 = 15;  // second gauge-converter warp (the first is warp 2)
+constexpr int kThreads = 640;
+constexpr int kEpiWG = 4;  // epilogue warpgroups
+constexpr int kConvWarp1 = 19;  // second gauge-converter warp (the first is warp 2)
 constexpr int kEpiWarp0 = 3;
 constexpr int kQCap = 20;  // repair jobs per warp and round
 constexpr int kAcc = 4;    // accumulator buffers in tensor memory
@@ -58,8 +60,8 @@ constexpr int kAcc = 4;    // accumulator buffers in tensor memory
 struct RowSmem {
     static constexpr uint32_t stages = 0;
     static constexpr uint32_t bsplit = stages + kStages * kTileBytes;  // 3 x (16 or 32 KB)
-    static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 12 warps x kQCap x 8 B
-    static constexpr uint32_t misc = queue + 12 * kQCap * 8;
+    static constexpr uint32_t queue = bsplit + kNPass * 32768;         // 16 warps x kQCap x 8 B
+    static constexpr uint32_t misc = queue + 4 * kEpiWG * kQCap * 8;
     static constexpr uint32_t total = misc + 512;  // base is 1024-aligned (checked in-kernel)
 };
 
@@ -335,8 +337,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
             }
             const float* Gf = a.G + tc::gauge_set(a, ti) * (int64_t)kD * g;
             if (cw == 0) prefetch_next_gauges(a, ti, g, lane);
-            convert_gauge_set<false, 2>(Gf, g, blk, NBK, fullk, bsz, bsplit, M->emaxb[ls & 3][cw], M->gmaxb[ls & 3][cw],
-                                        2 * cw, lane);
+            (void)convert_gauge_set<false, 2>(Gf, g, blk, NBK, fullk, bsz, bsplit, M->emaxb[ls & 3][cw],
+                                              M->gmaxb[ls & 3][cw], 2 * cw, lane);
             fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) mbar_arrive(&M->gready[ls & 3]);
@@ -345,7 +347,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
         }
     } else {
         // ------------------------------------------------------------ epilogue warpgroups
-        const int wg = (warp - kEpiWarp0) >> 2;  // warpgroup: tiles i = wg (mod 3)
+        const int wg = (warp - kEpiWarp0) >> 2;  // warpgroup: tiles i = wg (mod kEpiWG)
         const int q4 = warp & 3;                 // TMEM lane quadrant of this warp
         const int row = q4 * 32 + lane;          // TMEM lane = token row of the tile
         const int qw = warp - kEpiWarp0;         // job queue of this warp
@@ -356,7 +358,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
         int32_t flag = 0;
         tc::TileIter it;
         it.init(a, S, t_begin + wg);
-        for (int i = wg; i < my_tiles; i += 3, it.step(a, 3)) {
+        for (int i = wg; i < my_tiles; i += kEpiWG, it.step(a, kEpiWG)) {
             const tc::TileInfo ti = it.info(a);
             const int64_t ls = ti.seg - seg0;
             const int st = i % kStages, buf = i % kAcc;
@@ -430,13 +432,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
             }
 
             // ---- 3. error bound per block; scale/zero from the intervals when they agree
-            float E[NBK];
+            float E[NBK], Ec[NBK];  // Ec bounds |z~ - z|; E adds the rounding of the interval ends
             uint32_t s16[NBK], m16[NBK];
             int amb = 0;  // bit 2bk: scale needs the exact extremes; bit 2bk+1: zero needs the exact min
 #pragma unroll
             for (int bk = 0; bk < NBK; bk++) {
                 const float emax = fmaxf(M->emaxb[ls & 3][0][bk], M->emaxb[ls & 3][1][bk]);
-                E[bk] = sqrtf(nb[bk]) * 1.0001f * emax + (fabsf(mn[bk]) + fabsf(mx[bk])) * 2.4e-7f;
+                Ec[bk] = sqrtf(nb[bk]) * 1.0001f * emax;
+                E[bk] = Ec[bk] + (fabsf(mn[bk]) + fabsf(mx[bk])) * 2.4e-7f;
                 const float e = E[bk];
                 const float mn_lo = __fsub_rn(mn[bk], e), mn_hi = __fadd_rn(mn[bk], e);
                 const float mx_lo = __fsub_rn(mx[bk], e), mx_hi = __fadd_rn(mx[bk], e);
@@ -565,10 +568,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                     const float cc = -mz * r;
                     rinv[bk] = r;
                     c0[bk] = cc;
-                    // |t~ - t| <= E/s plus roundings: the fma and its inputs r and c0 (u|z r|,
+                    // |t~ - t| <= |z~ - z| / s plus roundings: the fma and its inputs r and c0 (u|z r|,
                     // 2u|c0|, u|t|) and the definition's subtract and divide (2u|t|)
                     const float zr = fmaxf(fabsf(mn[bk]), fabsf(mx[bk])) * r;
-                    const float mu = E[bk] * r * 1.0001f + (zr + 2.0f * fabsf(cc) + 3.0f * (qmaxf + 1.0f)) * 6.6e-8f;
+                    const float mu = Ec[bk] * r * 1.0001f + (zr + 2.0f * fabsf(cc) + 3.0f * (qmaxf + 1.0f)) * 6.6e-8f;
                     // mu < 1e-4: a code from z~ can only differ where the tolerance allows it
                     lim[bk] = mu < 0.99e-4f ? 2.0f : 0.5f - mu;
                     const float tlo = (mn[bk] - E[bk]) * r + cc, thi = (mx[bk] + E[bk]) * r + cc;

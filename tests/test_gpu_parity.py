@@ -229,3 +229,32 @@ def test_per_layer_calls_match_whole_call():
         cg.encode(shape1, params, dx[l * per_x:(l + 1) * per_x], dG[l * per_g:(l + 1) * per_g],
                   c2[l * nc1:(l + 1) * nc1], s2[l * ns1 // 4:(l + 1) * ns1 // 4], None)
     assert torch.equal(codes, c2) and torch.equal(scales, s2)
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("bu4_g128_blk64", dict(group=128, bits=4, block=64)),
+    ("bu6_g32_blk32", dict(group=32, bits=6, block=32)),
+    ("kivi3_g64", dict(backend=1, group=64, bits=3, block=128, residual=128)),
+])
+def test_many_tiles_per_cta(name, kw):
+    """Every CTA of the persistent tensor-core kernels walks tens of 128-token tiles and
+    several gauge changes (8 tiles per (layer, cache, head) set): the warpgroup rotation,
+    the accumulator and stage rings and the gauge conversion at each change, element by
+    element against the oracle."""
+    w = _wl(L=4, B=1, H=8, T=1024 + (128 if kw.get("backend") == 1 else 0), **kw)
+    x = synth.kv_cache(w, threads=8)
+    G = synth.gauges(w)
+    dx, dG = _dev(x, G)
+    shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
+    nc, ns, nr = cg.packed_bytes(shape, params)
+    codes, scales, resid = gpu_encode(w, dx, dG)
+    got = gpu_decode(w, codes, scales, resid, dG)
+    assert cg.get_status() == 0
+    ref = oracle.encode(w.shape, w.params, x, G, want_flags=True)
+    mism = compare_codes(w, _host_u8(codes, nc), ref["codes"], ref["flags"])
+    compare_scales(_host_u16(scales, ns), ref["scales"])
+    if nr:
+        np.testing.assert_array_equal(_host_u16(resid, nr), ref["residual"])
+    xr = oracle.decode(w.shape, w.params, ref["codes"], ref["scales"], ref["residual"], G)
+    step = scales_as_elements(w, ref["scales"]) * mism if mism.any() else None
+    compare_decode(w, got, xr, G, step)
