@@ -132,19 +132,17 @@ class Clocks:
 
 def _kernel_traffic(kind: str, workload: str):
     """ncu DRAM bytes (read + write) per launch of the kernel on this workload, recorded in
-    profiles/dram_traffic_<workload>.json, or None when there is no record or the kernel
-    source changed since the counters were taken."""
+    profiles/dram_traffic_<workload>.json, or None when there is no record or any source file
+    of the kernel changed since the counters were taken."""
     p = os.path.join(ROOT, "profiles", f"dram_traffic_{workload}.json")
     try:
         rec = json.load(open(p))[kind]
+        h = hashlib.sha256()
+        for name in rec["sources"]:
+            h.update(open(os.path.join(ROOT, "paper_2607_20538_gb300", "csrc", name), "rb").read())
     except Exception:
         return None
-    src = os.path.join(ROOT, "paper_2607_20538_gb300", "csrc", rec["source"])
-    try:
-        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
-    except Exception:
-        return None
-    return rec["bytes_per_launch"] if h == rec["source_sha"] else None
+    return rec["bytes_per_launch"] if h.hexdigest()[:16] == rec["sources_sha"] else None
 
 
 def cpu_sample(w, G, seconds=12.0, nthreads=None, start=0):
@@ -191,14 +189,23 @@ def workload_config(w, ws):
     return config
 
 
+def _workload(args):
+    """The workload of --workload, cut to --layers and with the --shape overrides."""
+    from paper_2607_20538_gb300 import synth
+    w = synth.WORKLOADS[args.workload]
+    if args.layers:
+        w = w.replace(L=min(args.layers, w.L))
+    if args.shape:
+        w = w.replace(**{k: int(v) for k, v in (kv.split("=") for kv in args.shape.split(","))})
+    return w
+
+
 def run_reference(args):
     ws, rank, _ = _dist()
     if rank != 0:
         return
     from paper_2607_20538_gb300 import synth
-    w = synth.WORKLOADS[args.workload]
-    if args.layers:
-        w = w.replace(L=min(args.layers, w.L))
+    w = _workload(args)
     G = synth.gauges(w)
     cores = os.cpu_count() or 1
     for i in range(args.warmup):
@@ -450,9 +457,7 @@ def run_cuda(args):
         torch.cuda.set_device(0)
     dev = torch.cuda.current_device()
     clock_dev = dev if ws == 1 else local
-    w = synth.WORKLOADS[args.workload]
-    if args.layers:
-        w = w.replace(L=min(args.layers, w.L))
+    w = _workload(args)
     stream = torch.cuda.current_stream()
     P = (_setup_rolling if w.T_cap else _setup_cache)(w, dev, ws, stream)
     t = _time_problem(P, stream, args.steps, args.warmup, dev, ws, clock_dev)
@@ -499,7 +504,7 @@ def run_cuda(args):
             "steps_per_s": round(1e3 / ms_step, 3),
             "roofline": {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 2), "peak": peak,
                          "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / peak, 4),
-                         "traffic": None if args.layers else _kernel_traffic(dom, w.name),
+                         "traffic": None if (args.layers or args.shape) else _kernel_traffic(dom, w.name),
                          "alg_bytes_per_launch": dom_alg,
                          "enc_frac": round(P.enc_alg / (enc_avg * 1e-3) / 1e9 / peak, 4),
                          "dec_frac": round(P.dec_alg / (dec_avg * 1e-3) / 1e9 / peak, 4)},
@@ -516,7 +521,7 @@ def run_cuda(args):
 
     # the other target workloads, device-timed in the same process (fewer steps)
     extra = {}
-    if not args.layers and not args.no_extra and args.workload == "llama3_8b":
+    if not args.layers and not args.shape and not args.no_extra and args.workload == "llama3_8b":
         for name in EXTRA_WORKLOADS:
             we = synth.WORKLOADS[name]
             Pe = (_setup_rolling if we.T_cap else _setup_cache)(we, dev, ws, stream)
@@ -557,6 +562,8 @@ def main():
     ap.add_argument("--workload", default="llama3_8b")
     ap.add_argument("--layers", type=int, default=0,
                     help="keep only the first N layers of the workload (small cases for profiling)")
+    ap.add_argument("--shape", default="",
+                    help="profiling slices: comma-separated workload overrides, e.g. L=1,d=256,T=32768")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--cpu-seconds-1t", type=float, default=4.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
