@@ -5,8 +5,8 @@ TEST INFRASTRUCTURE ONLY: imported by ``tests/``, ``__graft_entry__.smoke()`` an
 imports it. The arithmetic lives in ``cg_oracle.c`` (plain C, compiled with
 ``-ffp-contract=off`` and no fast-math); this module only marshals numpy arrays.
 
-Pins: ``tests/test_oracle_pins.py`` (closed forms, brute force, worked examples, library
-routines). No function here is "parity unpinned".
+Pins: ``tests/test_oracle_pins.py`` and ``tests/test_oracle_tile_pins.py`` (closed forms,
+brute force, worked examples, library routines). No function here is "parity unpinned".
 """
 from __future__ import annotations
 
@@ -20,7 +20,8 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libcgoracle.so")
 SRC_PATH = os.path.join(_HERE, "cg_oracle.c")
 
-BU, KIVI, NONE = 0, 1, 2
+BU, KIVI, NONE, TILE = 0, 1, 2, 3
+TILE_TOKENS = 16  # T_b: tokens per block-uniform tile (Sec. 4.2, Sec. 4.3)
 
 
 def build(force: bool = False) -> str:

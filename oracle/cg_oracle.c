@@ -18,9 +18,9 @@
  * Compiled without fast-math and with -ffp-contract=off, so every operation below is
  * the single IEEE operation it reads as.
  *
- * Status of the pins (tests/test_oracle_pins.py): every exported function is pinned
- * against closed forms, brute force, worked examples or library routines; none is
- * "parity unpinned".
+ * Status of the pins (tests/test_oracle_pins.py, tests/test_oracle_tile_pins.py): every
+ * exported function is pinned against closed forms, brute force, worked examples or
+ * library routines; none is "parity unpinned".
  */
 #include <math.h>
 #include <pthread.h>
@@ -32,7 +32,11 @@
 typedef struct { int32_t L, B, H, T, d, t0, T_cap; } cgo_shape;
 typedef struct { int32_t backend, group, bits, block, residual; } cgo_params;
 
-enum { CGO_BU = 0, CGO_KIVI = 1, CGO_NONE = 2 };
+enum { CGO_BU = 0, CGO_KIVI = 1, CGO_NONE = 2, CGO_BU_TILE = 3 };
+/* Block-uniform tile height: the paper partitions the token axis into blocks of T_b = 16
+ * tokens (Sec. 4.2, the value used for every checkpoint) and gives block-uniform one range
+ * per T_b x d_l block (Sec. 4.3). */
+enum { CGO_TILE_TOKENS = 16 };
 enum { CGO_OK = 0, CGO_EINVAL = -1, CGO_EUNSUP = -2, CGO_ERANGE = -4 };
 enum { CGO_FLAG_NONFINITE = 1, CGO_FLAG_FP16_OVERFLOW = 2 };
 
@@ -120,6 +124,11 @@ static int check_args(const cgo_shape* s, const cgo_params* p)
     if (p->backend == CGO_BU) {
         if (!valid_bits(p->bits) || p->block < 1 || s->d % p->block || (p->block * p->bits) % 8)
             return CGO_EINVAL;
+    } else if (p->backend == CGO_BU_TILE) {
+        if (!valid_bits(p->bits) || p->block < 1 || s->d % p->block || (p->block * p->bits) % 8)
+            return CGO_EINVAL;
+        /* a call starts at a tile boundary: a tile's range covers the tokens of one call */
+        if (s->t0 > 0 && s->t0 % CGO_TILE_TOKENS) return CGO_EUNSUP;
     } else if (p->backend == CGO_KIVI) {
         if (!valid_bits(p->bits) || p->block < 1 || s->d % p->block || (p->block * p->bits) % 8 ||
             p->residual < 0)
@@ -134,6 +143,7 @@ static int check_args(const cgo_shape* s, const cgo_params* p)
 }
 
 static int64_t tcap_of(const cgo_shape* s) { return s->T_cap ? s->T_cap : (int64_t)s->t0 + s->T; }
+static int64_t ntiles_of(const cgo_shape* s) { return (tcap_of(s) + CGO_TILE_TOKENS - 1) / CGO_TILE_TOKENS; }
 
 /* Measured bytes of each buffer (Appendix metric table: actual bits/value = measured
  * bytes / represented values), one count per stored item of the layouts. */
@@ -144,10 +154,12 @@ int cgo_packed_bytes(const cgo_shape* s, const cgo_params* p, int64_t* codes, in
     if (rc) return rc;
     int64_t units = (int64_t)s->L * 2 * s->B * s->H;
     int64_t d = s->d;
-    if (p->backend == CGO_BU) {
+    if (p->backend == CGO_BU || p->backend == CGO_BU_TILE) {
         int64_t tc = tcap_of(s), nb = d / p->block, pay = (int64_t)p->block * p->bits / 8;
+        /* one {scale, zero} pair per block of one token, or per block of one tile */
+        int64_t nranges = p->backend == CGO_BU ? tc : ntiles_of(s);
         *codes = units * tc * nb * pay;
-        *scales = units * tc * nb * 4;
+        *scales = units * nranges * nb * 4;
         *resid = 0;
     } else if (p->backend == CGO_KIVI) {
         int64_t nq = cgo_kivi_nq(s->T, p->residual, p->block);
@@ -382,6 +394,61 @@ static void bu_encode_unit(void* ctx, int64_t u)
     free(q);
 }
 
+/* ---- block-uniform tiles: one range per T_b x block tile (Sec. 4.3, T_b = 16 by Sec. 4.2) ----
+ * The tile's tokens are consecutive tokens of one (l, s, b, h); its range is the min/max of
+ * Z over all of them and the block's channels. Codes keep the per-token layout of the
+ * block-uniform rows; only the {scale, zero} pairs are per tile. The last tile of a call may
+ * hold fewer than T_b tokens; its range covers the tokens it holds. */
+static void tile_encode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group, blk = p->block, nb = d / blk, pay = blk * p->bits / 8;
+    int64_t h = u % s->H, sidx = (u / ((int64_t)s->H * s->B)) % 2, l = u / ((int64_t)s->H * s->B * 2);
+    const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+    int64_t tc = tcap_of(s), ntc = ntiles_of(s);
+    const int TB = CGO_TILE_TOKENS;
+    float* x = (float*)malloc(sizeof(float) * d);
+    float* zt = (float*)malloc(sizeof(float) * TB * d);   /* Z of the tile's tokens, [tt][c] */
+    float* v = (float*)malloc(sizeof(float) * TB * blk);  /* one tile block, [tt][c] */
+    uint8_t* q = (uint8_t*)malloc((size_t)TB * blk);
+    uint8_t* fl = (uint8_t*)malloc((size_t)TB * blk);
+    int st = 0;
+    for (int64_t ta = 0; ta < s->T; ta += TB) {
+        int nt = s->T - ta < TB ? (int)(s->T - ta) : TB;
+        for (int tt = 0; tt < nt; tt++) {
+            const uint16_t* xr = P->x + ((size_t)u * s->T + ta + tt) * d;
+            if (has_nonfinite(xr, d)) st |= CGO_FLAG_NONFINITE;
+            for (int c = 0; c < d; c++) x[c] = cgo_bf16_to_f32(xr[c]);
+            gauge_apply_f32(Gh, x, zt + (size_t)tt * d, d, g);
+            if (P->z_out) memcpy(P->z_out + ((size_t)u * s->T + ta + tt) * d, zt + (size_t)tt * d, sizeof(float) * d);
+        }
+        int64_t tile = (s->t0 + ta) / TB;
+        for (int b = 0; b < nb; b++) {
+            for (int tt = 0; tt < nt; tt++)
+                for (int c = 0; c < blk; c++) v[tt * blk + c] = zt[(size_t)tt * d + b * blk + c];
+            uint16_t s16, m16;
+            st |= quantize_block(v, nt * blk, 1, p->bits, &s16, &m16, q, P->flag_out ? fl : NULL, 1);
+            for (int tt = 0; tt < nt; tt++) {
+                int64_t th = s->t0 + ta + tt;
+                pack_codes(q + tt * blk, blk, p->bits, P->codes + (((size_t)u * tc + th) * nb + b) * pay);
+                if (P->flag_out)
+                    memcpy(P->flag_out + ((size_t)u * s->T + ta + tt) * d + (size_t)b * blk, fl + tt * blk, blk);
+            }
+            size_t rng_index = ((size_t)u * ntc + tile) * nb + b;
+            P->scales[rng_index * 2 + 0] = s16;
+            P->scales[rng_index * 2 + 1] = m16;
+        }
+    }
+    add_status(P, st);
+    free(x);
+    free(zt);
+    free(v);
+    free(q);
+    free(fl);
+}
+
 static void bu_decode_unit(void* ctx, int64_t u)
 {
     pool_t* P = (pool_t*)ctx;
@@ -402,9 +469,13 @@ static void bu_decode_unit(void* ctx, int64_t u)
             int nb = d / p->block, pay = p->block * p->bits / 8;
             for (int b = 0; b < nb; b++) {
                 size_t blk_index = ((size_t)u * tc + th) * nb + b;
+                /* the block's range: this token's own, or that of the tile holding it */
+                size_t rng_index = p->backend == CGO_BU_TILE
+                                       ? ((size_t)u * ntiles_of(s) + (size_t)(th / CGO_TILE_TOKENS)) * nb + b
+                                       : blk_index;
                 unpack_codes(P->in_codes + blk_index * pay, p->block, p->bits, q);
-                double sc = (double)cgo_f16_to_f32(P->in_scales[blk_index * 2 + 0]);
-                double mz = (double)cgo_f16_to_f32(P->in_scales[blk_index * 2 + 1]);
+                double sc = (double)cgo_f16_to_f32(P->in_scales[rng_index * 2 + 0]);
+                double mz = (double)cgo_f16_to_f32(P->in_scales[rng_index * 2 + 1]);
                 for (int k = 0; k < p->block; k++) zh[b * p->block + k] = (double)q[k] * sc + mz;
             }
         }
@@ -560,7 +631,7 @@ int cgo_encode(const cgo_shape* s, const cgo_params* p, const uint16_t* x, const
         P.fn = kivi_encode_unit;
     } else {
         P.n_units = (int64_t)s->L * 2 * s->B * s->H;
-        P.fn = bu_encode_unit;
+        P.fn = p->backend == CGO_BU_TILE ? tile_encode_unit : bu_encode_unit;
     }
     run_pool(&P, nthreads);
     if (status_out) *status_out = P.status;
