@@ -179,7 +179,7 @@ def cpu_sample(w, G, seconds=12.0, nthreads=None, start=0):
 def workload_config(w, ws):
     """The `config` of a bench line for workload `w` on `ws` ranks (both arms print the same)."""
     config = {"workload": w.name, "L": w.L, "B": w.B, "H": w.H, "T": w.T, "d": w.d,
-              "group": w.group, "backend": ["block-uniform", "kivi", "none"][w.backend],
+              "group": w.group, "backend": ["block-uniform", "kivi", "none", "block-uniform-tile"][w.backend],
               "bits": w.bits, "block": w.block, "residual": w.residual, "kv_dtype": "bf16",
               "parallelism": f"replicas{ws}", "l2": "inputs larger than L2 (no flush)",
               "value_def": "(bf16 bytes encoded + bf16 bytes decoded) / (encode+decode time)"}
@@ -438,7 +438,7 @@ PAPER_CONTEXT = {
 }
 
 # The other target workloads, timed in the same process after the headline one.
-EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling")
+EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "llama3_8b_tile")
 
 
 def run_cuda(args):

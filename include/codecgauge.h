@@ -33,6 +33,13 @@
  *   block-uniform (CG_BLOCK_UNIFORM), history of T_cap tokens:
  *     codes  : u8    [L][2][B][H][T_cap][d/block][block*bits/8]
  *     scales : half2 [L][2][B][H][T_cap][d/block]      .x = scale s, .y = zero (block min m)
+ *   block-uniform tiles (CG_BLOCK_TILE), T_b = CG_TILE_TOKENS, n_tiles = ceil(T_cap / T_b):
+ *     codes  : u8    [L][2][B][H][T_cap][d/block][block*bits/8]   (as CG_BLOCK_UNIFORM)
+ *     scales : half2 [L][2][B][H][n_tiles][d/block]  range of tokens [k T_b, (k+1) T_b) x block
+ *     A tile's range covers the tokens of the call that wrote it: the last tile of a call
+ *     may hold fewer than T_b tokens (its range covers those only), and a call starts at a
+ *     tile boundary (t0 % T_b == 0), so appending to an open tile means re-encoding it
+ *     from its first token.
  *   KIVI-style (CG_KIVI), n_q = max(0, floor((T - residual)/block)) * block quantized tokens:
  *     codes  per layer: keys  u8 [B][H][n_q/block][d][block*bits/8]   (per-channel token streams)
  *                       then values u8 [B][H][n_q][d/block][block*bits/8]
@@ -50,7 +57,8 @@
  *   z      = fp32 gauge-space value z_i = sum_j G[i][j] x_j in a fixed order: pairwise
  *            summation of the fp32 products G[i][j] * x_j (S(a,b) = S(a,m) + S(m,b),
  *            m = (a+b)/2, S(j,j+1) = the product), every product and sum rounded to fp32.
- *   s32    = (max - min) / (2^bits - 1) over the block (fp32 subtract, fp32 divide)
+ *   s32    = (max - min) / (2^bits - 1) over the block, or over the tile for
+ *            CG_BLOCK_TILE (fp32 subtract, fp32 divide)
  *   s, m   = fp16 round-to-nearest-even of s32 and of min; stored as half2 {s, m}
  *   q      = clamp(rint((z - m) / s), 0, 2^bits - 1)  (fp32; q = 0 when s == 0)
  *   decode : zhat = q * s + m ; xhat_i = sum_j G[j][i] zhat_j ; bf16 round-to-nearest-even.
@@ -72,10 +80,17 @@ extern "C" {
 #define CG_ECUDA        (-3)  /* a CUDA launch or runtime call failed; see cg_last_error()      */
 #define CG_ERANGE       (-4)  /* a byte count or index does not fit the library's integer types */
 
-/* Backends (Sec. 4.3 compression conditions; CG_NONE = the no-compression rows of Sec. 4.4). */
+/* Backends (Sec. 4.3 compression conditions; CG_NONE = the no-compression rows of Sec. 4.4).
+ * CG_BLOCK_TILE is block-uniform with one range per T_b x block tile, the block shape that
+ * Sec. 4.3 gives for block-uniform (T_b = 16 tokens, Sec. 4.2; block = d is its T_b x d_l
+ * tile); CG_BLOCK_UNIFORM takes one range per block of one token. */
 #define CG_BLOCK_UNIFORM 0
 #define CG_KIVI          1
 #define CG_NONE          2
+#define CG_BLOCK_TILE    3
+
+/* T_b: tokens per block-uniform tile (CG_BLOCK_TILE). */
+#define CG_TILE_TOKENS   16
 
 /* Device status bits, accumulated by kernels and read by cg_get_status(). */
 #define CG_FLAG_NONFINITE_INPUT 0x1  /* a NaN/Inf bf16 input value was seen                 */
@@ -84,9 +99,10 @@ extern "C" {
 
 /* Cache shape (Sec. 3 notation: B batch, H KV heads, T tokens, d head dimension, L layers).
  * d in {32, 64, 128, 256}; L*2*H <= 65535 and L*B*H <= 65535.
- * t0, T_cap: block-uniform only. Encode writes tokens [t0, t0+T) of a history that holds
- * T_cap tokens per (l, s, b, h); decode reads tokens [t0, t0+T) of it and writes a dense
- * [L][2][B][H][T][d] output. T_cap = 0 means T_cap = t0 + T. KIVI requires t0 = 0 and
+ * t0, T_cap: block-uniform (both kinds) only. Encode writes tokens [t0, t0+T) of a history
+ * that holds T_cap tokens per (l, s, b, h); decode reads tokens [t0, t0+T) of it and writes a
+ * dense [L][2][B][H][T][d] output. T_cap = 0 means T_cap = t0 + T. CG_BLOCK_TILE requires
+ * t0 % CG_TILE_TOKENS == 0 (CG_EUNSUPPORTED otherwise). KIVI requires t0 = 0 and
  * T_cap in {0, T}. */
 typedef struct {
     int32_t L, B, H, T, d;
@@ -94,12 +110,12 @@ typedef struct {
 } cg_shape;
 
 /* Codec parameters.
- *   backend  : CG_BLOCK_UNIFORM, CG_KIVI or CG_NONE
+ *   backend  : CG_BLOCK_UNIFORM, CG_BLOCK_TILE, CG_KIVI or CG_NONE
  *   group    : gauge group g (Sec. 3, R = d/g groups per head); g in {8,16,32,64,128}, d % g == 0
  *   bits     : 2, 3, 4, 6 or 8 (Sec. 4.3 bit settings; ignored by CG_NONE)
  *   block    : a power of two >= 8 with d % block == 0 and block*bits % 8 == 0;
- *              block-uniform: channels per block; KIVI: the key token-group length and
- *              the value channel-group length
+ *              block-uniform: channels per block (per tile for CG_BLOCK_TILE); KIVI: the
+ *              key token-group length and the value channel-group length
  *   residual : KIVI full-precision window length R >= 0 (ignored otherwise)           */
 typedef struct {
     int32_t backend;

@@ -16,10 +16,11 @@ import ctypes
 import os
 from dataclasses import dataclass
 
-__all__ = ["CG_BLOCK_UNIFORM", "CG_KIVI", "CG_NONE", "Shape", "Params", "packed_bytes", "encode", "decode",
-           "get_status", "lib_path", "load", "CodecGaugeError"]
+__all__ = ["CG_BLOCK_UNIFORM", "CG_KIVI", "CG_NONE", "CG_BLOCK_TILE", "CG_TILE_TOKENS", "Shape", "Params",
+           "packed_bytes", "encode", "decode", "get_status", "lib_path", "load", "CodecGaugeError"]
 
-CG_BLOCK_UNIFORM, CG_KIVI, CG_NONE = 0, 1, 2
+CG_BLOCK_UNIFORM, CG_KIVI, CG_NONE, CG_BLOCK_TILE = 0, 1, 2, 3
+CG_TILE_TOKENS = 16
 CG_FLAG_NONFINITE_INPUT, CG_FLAG_FP16_OVERFLOW, CG_FLAG_PIPE_TIMEOUT = 1, 2, 4
 _STATUS = {0: "CG_OK", -1: "CG_EINVAL", -2: "CG_EUNSUPPORTED", -3: "CG_ECUDA", -4: "CG_ERANGE"}
 

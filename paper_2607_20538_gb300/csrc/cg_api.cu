@@ -68,7 +68,7 @@ int status_ptr(int32_t** out) {
 }
 
 struct Sizes {
-    int64_t tcap, nq, nb, pay;
+    int64_t tcap, ntiles, nq, nb, pay;
     size_t codes, scales, resid;
     int64_t layer_codes, layer_scales, key_codes_per_bh, key_scales_per_bh, val_codes_per_bh, val_scales_per_bh;
 };
@@ -90,13 +90,21 @@ int validate(const cg_shape* sh, const cg_params* p, Sizes* z) {
     if (!(g == 8 || g == 16 || g == 32 || g == 64 || g == 128) || sh->d % g)
         return fail(CG_EINVAL, "group=%d: must be one of 8,16,32,64,128 and divide d=%d", g, sh->d);
     if (sh->t0 < 0 || sh->T_cap < 0) return fail(CG_EINVAL, "t0 and T_cap must be >= 0");
-    if (p->backend == CG_BLOCK_UNIFORM || p->backend == CG_KIVI) {
+    if (p->backend == CG_BLOCK_UNIFORM || p->backend == CG_KIVI || p->backend == CG_BLOCK_TILE) {
         if (!valid_bits(p->bits)) return fail(CG_EINVAL, "bits=%d: must be 2, 3, 4, 6 or 8", p->bits);
         if (!pow2(p->block) || p->block < 8 || sh->d % p->block)
             return fail(CG_EINVAL, "block=%d: must be a power of two >= 8 that divides d=%d", p->block, sh->d);
         if ((p->block * p->bits) % 8) return fail(CG_EINVAL, "block*bits must be a whole number of bytes");
     } else if (p->backend != CG_NONE) {
         return fail(CG_EINVAL, "unknown backend %d", p->backend);
+    }
+    if (p->backend == CG_BLOCK_TILE) {
+        if (sh->t0 % CG_TILE_TOKENS)
+            return fail(CG_EUNSUPPORTED, "block-uniform tiles: t0=%d must be a multiple of %d (a call re-encodes "
+                        "whole tiles)", sh->t0, CG_TILE_TOKENS);
+        if (tile_simt_smem(sh->d, g) == 0)
+            return fail(CG_EUNSUPPORTED, "block-uniform tiles: the gauge set of d=%d, group=%d does not fit one CTA",
+                        sh->d, g);
     }
     if (p->backend == CG_KIVI) {
         if (p->residual < 0) return fail(CG_EINVAL, "residual must be >= 0");
@@ -112,6 +120,7 @@ int validate(const cg_shape* sh, const cg_params* p, Sizes* z) {
         return fail(CG_ERANGE, "L*2*H and L*B*H must be <= 65535");
     const int64_t units = (int64_t)sh->L * 2 * sh->B * sh->H;
     z->tcap = tcap;
+    z->ntiles = (tcap + CG_TILE_TOKENS - 1) / CG_TILE_TOKENS;
     z->nq = 0;
     z->resid = 0;
     z->layer_codes = z->layer_scales = z->key_codes_per_bh = z->key_scales_per_bh = 0;
@@ -123,11 +132,12 @@ int validate(const cg_shape* sh, const cg_params* p, Sizes* z) {
         z->pay = 0;
         if (!mul_ok(rows, (size_t)sh->d * 4, &z->codes)) return fail(CG_ERANGE, "size overflow");
         z->scales = 0;
-    } else if (p->backend == CG_BLOCK_UNIFORM) {
+    } else if (p->backend == CG_BLOCK_UNIFORM || p->backend == CG_BLOCK_TILE) {
         z->nb = sh->d / p->block;
         z->pay = (int64_t)p->block * p->bits / 8;
         if (!mul_ok(rows, (size_t)(z->nb * z->pay), &z->codes)) return fail(CG_ERANGE, "size overflow");
-        if (!mul_ok(rows, (size_t)z->nb * 4, &z->scales)) return fail(CG_ERANGE, "size overflow");
+        const size_t nranges = p->backend == CG_BLOCK_UNIFORM ? rows : (size_t)units * (size_t)z->ntiles;
+        if (!mul_ok(nranges, (size_t)z->nb * 4, &z->scales)) return fail(CG_ERANGE, "size overflow");
     } else {
         const int64_t Gt = p->block, d = sh->d;
         z->nq = kivi_nq(sh->T, p->residual, Gt);
@@ -148,8 +158,11 @@ int validate(const cg_shape* sh, const cg_params* p, Sizes* z) {
     return CG_OK;
 }
 
-// Row map for the block-uniform / none history layout [L][2][B][H][T_cap][...].
-void bu_maps(const cg_shape* sh, const Sizes& z, int64_t rowbytes, int64_t rowscales, RowMap* cm, RowMap* sm) {
+// Row map for the block-uniform / none history layout [L][2][B][H][T_cap][...]. With
+// tile = true the scales are per 16-token tile, [L][2][B][H][ceil(T_cap/16)][d/block]
+// (t0 is then a multiple of 16).
+void bu_maps(const cg_shape* sh, const Sizes& z, int64_t rowbytes, int64_t rowscales, RowMap* cm, RowMap* sm,
+             bool tile = false) {
     const int64_t tc = z.tcap;
     cm->sT = rowbytes;
     cm->sH = tc * rowbytes;
@@ -157,12 +170,15 @@ void bu_maps(const cg_shape* sh, const Sizes& z, int64_t rowbytes, int64_t rowsc
     cm->sS = (int64_t)sh->B * cm->sB;
     cm->sL = 2 * cm->sS;
     cm->base = (int64_t)sh->t0 * rowbytes;
+    cm->tshift = 0;
+    const int64_t nranges = tile ? z.ntiles : tc;
     sm->sT = rowscales;
-    sm->sH = tc * rowscales;
+    sm->sH = nranges * rowscales;
     sm->sB = (int64_t)sh->H * sm->sH;
     sm->sS = (int64_t)sh->B * sm->sB;
     sm->sL = 2 * sm->sS;
-    sm->base = (int64_t)sh->t0 * rowscales;
+    sm->tshift = tile ? 4 : 0;
+    sm->base = (int64_t)(sh->t0 >> sm->tshift) * rowscales;
 }
 
 // Row map for KIVI keys seen as rows of the key tensor: codes [B][H][n_q/Gt][d][pay] at the
@@ -176,7 +192,9 @@ void kivi_key_maps(const cg_shape* sh, const cg_params* p, const Sizes& z, RowMa
     cm->sH = z.key_codes_per_bh;
     cm->sB = (int64_t)sh->H * cm->sH;
     cm->sT = (int64_t)sh->d * z.pay / Gt;
+    cm->tshift = 0;
     sm->base = 0;
+    sm->tshift = 0;
     sm->sL = z.layer_scales;
     sm->sS = 0;
     sm->sH = z.key_scales_per_bh;
@@ -193,7 +211,9 @@ void kivi_value_maps(const cg_shape* sh, const Sizes& z, RowMap* cm, RowMap* sm)
     cm->sS = 0;
     cm->sL = z.layer_codes;
     cm->base = BH * z.key_codes_per_bh;
+    cm->tshift = 0;
     sm->sT = z.nb;
+    sm->tshift = 0;
     sm->sH = z.val_scales_per_bh;
     sm->sB = (int64_t)sh->H * sm->sH;
     sm->sS = 0;
@@ -279,6 +299,7 @@ CG_EXPORT int cg_encode(const cg_shape* shape, const cg_params* params, const vo
     int rc = validate(shape, params, &z);
     if (rc) return rc;
     const bool kivi = params->backend == CG_KIVI, none = params->backend == CG_NONE;
+    const bool tile = params->backend == CG_BLOCK_TILE;
     if (shape->T == 0) return CG_OK;
     if (!kv_bf16 || !gauges) return fail(CG_EINVAL, "null kv or gauges pointer");
     if (z.codes && !out_codes) return fail(CG_EINVAL, "null out_codes");
@@ -296,6 +317,12 @@ CG_EXPORT int cg_encode(const cg_shape* shape, const cg_params* params, const vo
     a.G = gauges;
     a.codes = static_cast<uint8_t*>(out_codes);
     a.scales = static_cast<uint32_t*>(out_scales);
+    if (tile) {
+        bu_maps(shape, z, z.nb * z.pay, z.nb, &a.cmap, &a.smap, true);
+        e = launch_tile_encode_simt(a, st);
+        if (e != cudaSuccess) return cuda_fail(e, "tile encode launch");
+        return CG_OK;
+    }
     if (!kivi) {
         bu_maps(shape, z, none ? (int64_t)shape->d * 4 : z.nb * z.pay, z.nb, &a.cmap, &a.smap);
         if (!none && tc_row_encode_eligible(a)) {
@@ -352,6 +379,7 @@ CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const vo
     int rc = validate(shape, params, &z);
     if (rc) return rc;
     const bool kivi = params->backend == CG_KIVI, none = params->backend == CG_NONE;
+    const bool tile = params->backend == CG_BLOCK_TILE;
     if (shape->T == 0) return CG_OK;
     if (!out_kv_bf16 || !gauges) return fail(CG_EINVAL, "null output or gauges pointer");
     if (z.codes && !codes) return fail(CG_EINVAL, "null codes");
@@ -370,7 +398,7 @@ CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const vo
     a.codes = const_cast<uint8_t*>(static_cast<const uint8_t*>(codes));
     a.scales = const_cast<uint32_t*>(static_cast<const uint32_t*>(scales));
     if (!kivi) {
-        bu_maps(shape, z, none ? (int64_t)shape->d * 4 : z.nb * z.pay, z.nb, &a.cmap, &a.smap);
+        bu_maps(shape, z, none ? (int64_t)shape->d * 4 : z.nb * z.pay, z.nb, &a.cmap, &a.smap, tile);
         if (!none && tc_row_decode_eligible(a)) {
             e = tc_launch_row_decode(a, st);
         } else {

@@ -80,11 +80,13 @@ __host__ __device__ __forceinline__ int64_t kivi_nq(int64_t T, int64_t R, int64_
 }
 
 // Byte/element strides that place one row (one token of one (l, s, b, h)) of the packed
-// outputs; row offset = base + l*sL + s*sS + b*sB + h*sH + t*sT.
+// outputs; row offset = base + l*sL + s*sS + b*sB + h*sH + (t >> tshift)*sT. A shift of 4
+// maps the 16 tokens of a block-uniform tile to the tile's one set of scales.
 struct RowMap {
     int64_t base, sL, sS, sB, sH, sT;
+    int tshift;
     __host__ __device__ __forceinline__ int64_t at(int l, int s, int b, int h, int64_t t) const {
-        return base + l * sL + s * sS + b * sB + h * sH + t * sT;
+        return base + l * sL + s * sS + b * sB + h * sH + (t >> tshift) * sT;
     }
 };
 

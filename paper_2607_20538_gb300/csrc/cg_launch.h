@@ -52,12 +52,14 @@ struct ResidArgs {
 
 cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st);
+cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st);
 cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st);
 cudaError_t launch_residual_copy(const ResidArgs& a, cudaStream_t st);
 
 // Shared-memory bytes the SIMT kernels need (0 = shape not supported by them).
 size_t row_simt_smem(int d, int g);
+size_t tile_simt_smem(int d, int g);
 size_t key_simt_smem(int d, int g, int Gt, int bits);
 
 }  // namespace cg

@@ -185,6 +185,190 @@ __global__ void __launch_bounds__(kRowThreads) row_encode_kernel(RowArgs a) {
 }
 
 // ------------------------------------------------------------------------------------
+// Block-uniform tiles: Z = G X for the 16 tokens of a tile, then one min/max range per
+// tile block (16 tokens x blk channels, Sec. 4.3 with T_b = 16 from Sec. 4.2), codes and
+// packing in the per-token row layout, one {scale, zero} pair per tile block.
+// One warp per tile; the CTA shares the (l, s, h) gauge set in shared memory.
+// ------------------------------------------------------------------------------------
+constexpr int kTileTokens = CG_TILE_TOKENS;
+constexpr int kTileWarpsMax = 16;
+constexpr size_t kSmemOptIn = 232448;  // 227 KB of dynamic shared memory per CTA
+
+__host__ __device__ __forceinline__ size_t tile_warp_bytes(int d) {
+    return (size_t)kTileTokens * d * 4 + (size_t)kTileTokens * d + 32 * 4;
+}
+
+// Binary-carry merge of the chunk sums of one pairwise sum (see gauge_coord).
+__device__ __forceinline__ void carry_push(float& l0, float& l1, float& l2, float& l3, float& v, int c) {
+    if (c & 1) {
+        v = __fadd_rn(l0, v);
+        if (c & 2) {
+            v = __fadd_rn(l1, v);
+            if (c & 4) {
+                v = __fadd_rn(l2, v);
+                if (c & 8) v = __fadd_rn(l3, v);
+                else l3 = v;
+            } else {
+                l2 = v;
+            }
+        } else {
+            l1 = v;
+        }
+    } else {
+        l0 = v;
+    }
+}
+
+// gauge_coord for four tokens at once: out[t] = sum_j G[i][j] x_t[j] in the library's
+// pairwise order, x_t = x0 + t * xstride (16-byte aligned rows). Each gauge value loaded
+// from shared memory serves the four tokens.
+__device__ __forceinline__ void gauge_coord4(const float* Gcol, int gstride, const float* x0, int xstride, int g,
+                                             float (&out)[4]) {
+    float l0[4] = {}, l1[4] = {}, l2[4] = {}, l3[4] = {}, v[4] = {};
+#pragma unroll 1
+    for (int c = 0; c < g / 8; c++) {
+        float a[8];
+#pragma unroll
+        for (int k = 0; k < 8; k++) a[k] = Gcol[(8 * c + k) * gstride];
+#pragma unroll
+        for (int t = 0; t < 4; t++) {
+            const float4* xp = reinterpret_cast<const float4*>(x0 + t * xstride + 8 * c);
+            const float4 u0 = xp[0], u1 = xp[1];
+            const float b[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+            v[t] = tree8(a, b);
+            carry_push(l0[t], l1[t], l2[t], l3[t], v[t], c);
+        }
+    }
+#pragma unroll
+    for (int t = 0; t < 4; t++) out[t] = v[t];
+}
+
+template <int NR>
+__global__ void __launch_bounds__(kTileWarpsMax * 32) tile_encode_kernel(RowArgs a) {
+    constexpr int d = NR * 32;
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int g = a.g;
+    float* Gs = reinterpret_cast<float*>(smem);  // Gs[r][jj][i] = G_r[i][jj]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+    unsigned char* wbase = smem + (size_t)d * g * 4 + (size_t)warp * tile_warp_bytes(d);
+    float* buf = reinterpret_cast<float*>(wbase);                         // [16][d]: x, then z
+    uint8_t* qs = wbase + (size_t)kTileTokens * d * 4;                    // [16][d] codes
+    uint32_t* smw = reinterpret_cast<uint32_t*>(qs + (size_t)kTileTokens * d);  // [d/blk] scales
+
+    const int y = blockIdx.y;
+    const int h = y % a.H;
+    const int s = a.s_lo + (y / a.H) % a.s_n;
+    const int l = y / (a.H * a.s_n);
+    const float* Gsrc = a.G + ((int64_t)(l * 2 + s) * a.H + h) * (int64_t)d * g;
+    for (int e = threadIdx.x; e < d * g; e += blockDim.x) {
+        int r = e / (g * g), rem = e - r * g * g, i = rem / g, jj = rem - i * g;
+        Gs[r * g * g + jj * g + i] = __ldg(Gsrc + e);
+    }
+    __syncthreads();
+
+    const int64_t ntc = (a.t_count + kTileTokens - 1) / kTileTokens;  // tiles per unit in this call
+    const int64_t total = (int64_t)a.B * ntc;
+    const int64_t chunk = (total + gridDim.x - 1) / gridDim.x;
+    const int64_t k0 = (int64_t)blockIdx.x * chunk;
+    const int64_t k1 = k0 + chunk < total ? k0 + chunk : total;
+    const int bits = a.bits, blk = a.blk;
+    const int qmax = (1 << bits) - 1;
+    const float qmaxf = (float)qmax;
+    const int nw = d * bits / 32;  // packed words per token row
+    int32_t flag = 0;
+
+    for (int64_t tk = k0 + warp; tk < k1; tk += nwarps) {
+        const int b = (int)(tk / ntc);
+        const int64_t t_lo = (tk - (int64_t)b * ntc) * kTileTokens;
+        const int nt = a.t_count - t_lo < kTileTokens ? (int)(a.t_count - t_lo) : kTileTokens;
+        // the tile's tokens are nt consecutive rows of x: nt * d bf16, 16-byte chunks
+        const uint4* xt = reinterpret_cast<const uint4*>(
+            a.x + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t_lo) * d);
+        for (int e = lane; e < nt * d / 8; e += 32) {
+            const uint4 v = __ldg(xt + e);
+            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            float f[8];
+#pragma unroll
+            for (int k = 0; k < 4; k++) {
+                const uint32_t lo = w[k] & 0xffffu, hi = w[k] >> 16;
+                if (bf16_nonfinite(lo) || bf16_nonfinite(hi)) flag |= CG_FLAG_NONFINITE_INPUT;
+                f[2 * k] = bf16_bits_to_float(lo);
+                f[2 * k + 1] = bf16_bits_to_float(hi);
+            }
+            float4* dst = reinterpret_cast<float4*>(buf + 8 * e);
+            dst[0] = make_float4(f[0], f[1], f[2], f[3]);
+            dst[1] = make_float4(f[4], f[5], f[6], f[7]);
+        }
+        __syncwarp();
+        // Z for four tokens at a time; each quad's z overwrites its x rows once all lanes
+        // have read them
+        for (int tq = 0; tq * 4 < nt; tq++) {
+            float zq[NR][4];
+#pragma unroll
+            for (int k = 0; k < NR; k++) {
+                const int c = lane + 32 * k, r = c / g, i = c - r * g;
+                gauge_coord4(Gs + r * g * g + i, g, buf + (size_t)(4 * tq) * d + r * g, d, g, zq[k]);
+            }
+            __syncwarp();
+#pragma unroll
+            for (int t = 0; t < 4; t++)
+                if (4 * tq + t < nt) {
+#pragma unroll
+                    for (int k = 0; k < NR; k++) buf[(4 * tq + t) * d + lane + 32 * k] = zq[k][t];
+                }
+            __syncwarp();
+        }
+        // tile block ranges: tokens per lane, then lanes (segments of min(blk, 32)), then
+        // registers for blk > 32
+        const int seg = blk < 32 ? blk : 32;
+        const int per = blk > 32 ? blk / 32 : 1;
+        float mn[NR], mx[NR];
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k;
+            float lo = buf[c], hi = lo;
+            for (int tt = 1; tt < nt; tt++) {
+                const float v = buf[tt * d + c];
+                lo = fminf(lo, v);
+                hi = fmaxf(hi, v);
+            }
+            mn[k] = seg_min(lo, seg);
+            mx[k] = seg_max(hi, seg);
+        }
+        if (per > 1) {
+#pragma unroll
+            for (int k = 0; k < NR; k++) {
+                const int kb = (k / per) * per;
+                float a0 = mn[kb], a1 = mx[kb];
+                for (int kk = 1; kk < per; kk++) {
+                    a0 = fminf(a0, mn[kb + kk]);
+                    a1 = fmaxf(a1, mx[kb + kk]);
+                }
+                mn[k] = a0;
+                mx[k] = a1;
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < NR; k++) {
+            const int c = lane + 32 * k;
+            const uint32_t sz = scale_zero(mn[k], mx[k], qmaxf, &flag);
+            const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
+            for (int tt = 0; tt < nt; tt++) qs[tt * d + c] = (uint8_t)quant_code(buf[tt * d + c], sc, mz, qmax);
+            if ((c % blk) == 0) smw[c / blk] = sz;
+        }
+        __syncwarp();
+        for (int e = lane; e < nt * nw; e += 32) {
+            const int tt = e / nw, w = e - tt * nw;
+            uint32_t* cw = reinterpret_cast<uint32_t*>(a.codes + a.cmap.at(l, s, b, h, t_lo + tt));
+            cw[w] = pack_word(qs + tt * d, w, bits);
+        }
+        if (lane < d / blk) a.scales[a.smap.at(l, s, b, h, t_lo) + lane] = smw[lane];
+        __syncwarp();
+    }
+    if (flag) raise_flag(a.status, flag);
+}
+
+// ------------------------------------------------------------------------------------
 // Row decode: unpack, dequantize zhat = q*s + m, then Xhat = G^T Zhat, bf16 store.
 // ------------------------------------------------------------------------------------
 template <int NR>
@@ -390,6 +574,20 @@ __global__ void residual_copy_kernel(ResidArgs a) {
 
 }  // namespace
 
+// Warps per CTA of the tile encode kernel: as many as shared memory holds, at most 16.
+static int tile_simt_warps(int d, int g) {
+    if (!(d == 32 || d == 64 || d == 128 || d == 256)) return 0;
+    const size_t gbytes = (size_t)d * g * 4;
+    if (gbytes >= kSmemOptIn) return 0;
+    const size_t n = (kSmemOptIn - gbytes) / tile_warp_bytes(d);
+    return n < (size_t)kTileWarpsMax ? (int)n : kTileWarpsMax;
+}
+
+size_t tile_simt_smem(int d, int g) {
+    const int nw = tile_simt_warps(d, g);
+    return nw < 1 ? 0 : (size_t)d * g * 4 + (size_t)nw * tile_warp_bytes(d);
+}
+
 size_t row_simt_smem(int d, int g) {
     if (!(d == 32 || d == 64 || d == 128 || d == 256)) return 0;
     size_t enc = (size_t)d * g * 4 + (size_t)kRowWarps * d * 5 + (size_t)kRowWarps * 32 * 4;
@@ -412,6 +610,22 @@ static cudaError_t row_encode_nr(const RowArgs& a, cudaStream_t st) {
     if (e != cudaSuccess) return e;
     dim3 grid((unsigned)((a.B * a.t_count + kRowsPerCta - 1) / kRowsPerCta), (unsigned)(a.L * a.s_n * a.H));
     row_encode_kernel<NR><<<grid, kRowThreads, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+template <int NR>
+static cudaError_t tile_encode_nr(const RowArgs& a, cudaStream_t st) {
+    const int nwarps = tile_simt_warps(a.d, a.g);
+    const size_t smem = tile_simt_smem(a.d, a.g);
+    if (nwarps < 1) return cudaErrorInvalidValue;
+    cudaError_t e = cudaFuncSetAttribute(tile_encode_kernel<NR>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    // two tiles per warp per CTA; the tiles of one (l, s, h) spread over grid.x
+    const int64_t tiles = (int64_t)a.B * ((a.t_count + kTileTokens - 1) / kTileTokens);
+    int64_t gx = (tiles + 2 * nwarps - 1) / (2 * nwarps);
+    if (gx > 65535) gx = 65535;
+    dim3 grid((unsigned)gx, (unsigned)(a.L * a.s_n * a.H));
+    tile_encode_kernel<NR><<<grid, nwarps * 32, smem, st>>>(a);
     return cudaGetLastError();
 }
 
@@ -456,6 +670,7 @@ static cudaError_t key_decode_nr(const KeyArgs& a, cudaStream_t st) {
 
 cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_encode_nr, a.d, a, st) }
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_decode_nr, a.d, a, st) }
+cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(tile_encode_nr, a.d, a, st) }
 cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_encode_nr, a.d, a, st) }
 cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_decode_nr, a.d, a, st) }
 

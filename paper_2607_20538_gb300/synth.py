@@ -38,7 +38,7 @@ class Workload:
     T: int
     d: int
     group: int
-    backend: int          # 0 block-uniform, 1 KIVI, 2 none
+    backend: int          # 0 block-uniform, 1 KIVI, 2 none, 3 block-uniform tiles
     bits: int
     block: int
     residual: int = 0
@@ -69,8 +69,9 @@ class Workload:
         return Workload(**d)
 
 
-# The five cache workloads: a tiny case, a Llama-3-8B-shaped cache, a Qwen/Mistral-shaped
-# KIVI case, a Gemma-2-27B-shaped 6-bit case and a rolling decode step over a 16k history.
+# The cache workloads: a tiny case, a Llama-3-8B-shaped cache (per-token blocks, and the
+# paper's 16-token tiles), a Qwen/Mistral-shaped KIVI case, a Gemma-2-27B-shaped 6-bit case
+# and a rolling decode step over a 16k history.
 WORKLOADS = {
     "tiny": Workload("tiny", L=1, B=1, H=2, T=256, d=64, group=16, backend=0, bits=4, block=32,
                      n_outlier=2, outlier_mult=10.0, sigma_v=0.3, kv_seed=1000, gauge_seed=2000),
@@ -83,6 +84,10 @@ WORKLOADS = {
     "gemma27b": Workload("gemma27b", L=46, B=2, H=16, T=8192, d=128, group=32, backend=0, bits=6,
                          block=32, n_outlier=8, outlier_mult=20.0, sigma_v=0.5, kv_seed=1003,
                          gauge_seed=2003),
+    # the paper's block-uniform block shape on the 8B cache: one range per 16-token x d tile
+    "llama3_8b_tile": Workload("llama3_8b_tile", L=32, B=1, H=8, T=8192, d=128, group=128, backend=3,
+                               bits=4, block=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,
+                               kv_seed=1001, gauge_seed=2001),
     # rolling: history of T_cap=16384 tokens; T is the decode length of one step
     "rolling": Workload("rolling", L=32, B=64, H=8, T=16384, d=128, group=128, backend=0, bits=4,
                         block=64, n_outlier=4, outlier_mult=10.0, sigma_v=0.3, kv_seed=1004,

@@ -35,7 +35,7 @@ def codes_as_elements(w, codes: np.ndarray, T: int | None = None) -> np.ndarray:
     """Codes laid out like the cache, [L][2][B][H][T][d] (KIVI residual tokens = 0)."""
     T = w.T if T is None else T
     L, B, H, d, bits = w.L, w.B, w.H, w.d, w.bits
-    if w.backend == 0:
+    if w.backend in (0, 3):  # block-uniform rows and tiles share the per-token code layout
         q = unpack_stream(codes, L * 2 * B * H * T * d, bits)
         return q.reshape(L, 2, B, H, T, d)
     Gt = w.block
@@ -61,6 +61,10 @@ def scales_as_elements(w, scales_u16: np.ndarray, T: int | None = None, which: i
     if w.backend == 0:
         nb = d // w.block
         return np.repeat(s.reshape(L, 2, B, H, T, nb), w.block, axis=-1)
+    if w.backend == 3:  # one pair per 16-token tile block
+        nb, TB = d // w.block, oracle.TILE_TOKENS
+        st = s.reshape(L, 2, B, H, -1, nb)[:, :, :, :, np.arange(T) // TB, :]
+        return np.repeat(st, w.block, axis=-1)
     Gt = w.block
     nq = oracle.kivi_nq(T, w.residual, Gt)
     out = np.zeros((L, 2, B, H, T, d), np.float32)

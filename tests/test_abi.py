@@ -43,8 +43,8 @@ def test_exports_every_declared_symbol(lib):
 def test_packed_bytes_match_oracle(lib, name):
     w = synth.WORKLOADS[name]
     assert cg.packed_bytes(cg.Shape(**w.shape), cg.Params(**w.params)) == oracle.packed_bytes(w.shape, w.params)
-    for backend in (0, 1, 2):
-        for T in (0, 1, 127, 128, 129, 300):
+    for backend in (0, 1, 2, 3):
+        for T in (0, 1, 15, 16, 17, 127, 128, 129, 300):
             ww = w.replace(backend=backend, T=T, T_cap=0, L=2, B=2, H=3)
             assert cg.packed_bytes(cg.Shape(**ww.shape), cg.Params(**ww.params)) == \
                 oracle.packed_bytes(ww.shape, ww.params)
@@ -68,6 +68,21 @@ def test_validation(lib, bad):
         cg.packed_bytes(shape, params)
     assert e.value.code in (-1, -2)
     assert lib.cg_last_error().decode()
+
+
+def test_tile_history_offsets(lib):
+    """Block-uniform tiles: a call starts at a tile boundary (t0 % 16 == 0); the scales of a
+    T_cap history are one pair per tile block, as the oracle counts them."""
+    params = cg.Params(cg.CG_BLOCK_TILE, 32, 4, 64)
+    for t0, T, T_cap, ok in ((0, 5, 40, True), (16, 9, 40, True), (32, 8, 40, True), (8, 4, 40, False),
+                             (17, 1, 40, False), (16, 30, 40, False)):
+        sh = dict(L=1, B=2, H=3, T=T, d=128, t0=t0, T_cap=T_cap)
+        if ok:
+            assert cg.packed_bytes(cg.Shape(**sh), params) == oracle.packed_bytes(sh, params.__dict__)
+        else:
+            with pytest.raises(cg.CodecGaugeError) as e:
+                cg.packed_bytes(cg.Shape(**sh), params)
+            assert e.value.code == (-1 if t0 + T > T_cap else -2)
 
 
 def test_pointer_checks_fail_before_device(lib):

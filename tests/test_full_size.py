@@ -1,4 +1,4 @@
-"""Full-size parity: the four large cache workloads, encoded and decoded by whole-workload
+"""Full-size parity: the large cache workloads, encoded and decoded by whole-workload
 calls (the launch configuration the benchmark times), checked against the oracle on sampled
 (layer, batch, head) units, keys and values.
 
@@ -68,7 +68,7 @@ def _release_device_memory():
     torch.cuda.empty_cache()
 
 
-@pytest.mark.parametrize("name", ["llama3_8b", "gemma27b", "kivi3_qwen"])
+@pytest.mark.parametrize("name", ["llama3_8b", "gemma27b", "kivi3_qwen", "llama3_8b_tile"])
 def test_full_size_sampled(name):
     w = synth.WORKLOADS[name]
     x = synth.kv_cache(w, threads=16)
@@ -88,9 +88,14 @@ def test_full_size_sampled(name):
     for (l, b, h) in _units(w):
         xu = np.ascontiguousarray(x[l:l + 1, :, b:b + 1, h:h + 1])
         ou = o16.view(w.L, 2, w.B, w.H, w.T, w.d)[l, :, b, h].contiguous().cpu().numpy().view(np.uint16).ravel()
-        if w.backend == 0:
+        if w.backend in (0, 3):
             cu = _sub_bu(c8, w, w.T, l, b, h, w.d * w.bits // 8)
-            su = _sub_bu(s32, w, w.T, l, b, h, w.d // w.block).view(np.uint16)
+            if w.backend == 0:
+                su = _sub_bu(s32, w, w.T, l, b, h, w.d // w.block).view(np.uint16)
+            else:  # one pair per 16-token tile block
+                nt = -(-w.T // oracle.TILE_TOKENS)
+                su = s32.view(w.L, 2, w.B, w.H, nt, w.d // w.block)[l, :, b, h].contiguous().cpu().numpy()
+                su = su.ravel().view(np.uint16)
             ru = np.zeros(0, np.uint16)
         else:
             nq = oracle.kivi_nq(w.T, w.residual, w.block)
