@@ -5,7 +5,8 @@ TEST INFRASTRUCTURE ONLY: imported by ``tests/``, ``__graft_entry__.smoke()`` an
 imports it. The arithmetic lives in ``cg_oracle.c`` (plain C, compiled with
 ``-ffp-contract=off`` and no fast-math); this module only marshals numpy arrays.
 
-Pins: ``tests/test_oracle_pins.py`` and ``tests/test_oracle_tile_pins.py`` (closed forms,
+Pins: ``tests/test_oracle_pins.py``, ``tests/test_oracle_tile_pins.py`` and
+``tests/test_oracle_stream_pins.py`` (closed forms,
 brute force, worked examples, library routines). No function here is "parity unpinned".
 """
 from __future__ import annotations
@@ -69,6 +70,13 @@ def lib():
         L.cgo_pack.argtypes = [vp, ctypes.c_int, ctypes.c_int, vp]
         L.cgo_unpack.restype = None
         L.cgo_unpack.argtypes = [vp, ctypes.c_int, ctypes.c_int, vp]
+        L.cgo_kivi_stream_bytes.restype = ctypes.c_int
+        L.cgo_kivi_stream_bytes.argtypes = [P(_Shape), P(_Params), P(ctypes.c_int64), P(ctypes.c_int64),
+                                            P(ctypes.c_int64)]
+        L.cgo_kivi_append.restype = ctypes.c_int
+        L.cgo_kivi_append.argtypes = [P(_Shape), P(_Params), vp, vp, vp, vp, vp, ctypes.c_int, P(ctypes.c_int32)]
+        L.cgo_kivi_stream_decode.restype = ctypes.c_int
+        L.cgo_kivi_stream_decode.argtypes = [P(_Shape), P(_Params), vp, vp, vp, vp, vp, ctypes.c_int]
         L.cgo_gauge_coord.restype = ctypes.c_float
         L.cgo_gauge_coord.argtypes = [vp, vp, ctypes.c_int]
         _lib = L
@@ -162,4 +170,56 @@ def decode(shape: dict, params: dict, codes, scales, residual, gauges, *, nthrea
                           _ptr(scales), _ptr(residual), _ptr(G), _ptr(out), nthreads or (os.cpu_count() or 1))
     if rc:
         raise ValueError(f"oracle decode rc={rc}")
+    return out
+
+
+# ---------------------------------------------------------------- KIVI streaming
+def kivi_stream_bytes(shape: dict, params: dict):
+    """(codes, scales, ring) bytes of a KIVI stream of capacity shape["T_cap"]."""
+    c, s, r = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_int64()
+    sh = dict(t0=0, T_cap=0)
+    sh.update(shape)
+    rc = lib().cgo_kivi_stream_bytes(ctypes.byref(_shape(**sh)), ctypes.byref(_Params(**params)),
+                                     ctypes.byref(c), ctypes.byref(s), ctypes.byref(r))
+    if rc:
+        raise ValueError(f"oracle kivi_stream_bytes rc={rc}")
+    return c.value, s.value, r.value
+
+
+def kivi_stream_alloc(shape: dict, params: dict):
+    """Zeroed stream buffers (codes u8, scales u16 pairs, ring u16) for capacity shape["T_cap"]."""
+    nc, ns, nr = kivi_stream_bytes(shape, params)
+    return np.zeros(nc, np.uint8), np.zeros(ns // 2, np.uint16), np.zeros(nr // 2, np.uint16)
+
+
+def kivi_append(shape: dict, params: dict, x_new: np.ndarray, gauges: np.ndarray, codes, scales, ring,
+                *, nthreads: int = 0) -> int:
+    """Append tokens [t0, t0 + T) to the stream buffers in place; returns the status bits."""
+    sh = dict(t0=0, T_cap=0)
+    sh.update(shape)
+    x = np.ascontiguousarray(x_new).view(np.uint16)
+    assert x.size == sh["L"] * 2 * sh["B"] * sh["H"] * sh["T"] * sh["d"]
+    G = np.ascontiguousarray(gauges, np.float32)
+    st = ctypes.c_int32(0)
+    rc = lib().cgo_kivi_append(ctypes.byref(_shape(**sh)), ctypes.byref(_Params(**params)), _ptr(x), _ptr(G),
+                               _ptr(codes), _ptr(scales), _ptr(ring), nthreads or (os.cpu_count() or 1),
+                               ctypes.byref(st))
+    if rc:
+        raise ValueError(f"oracle kivi_append rc={rc}")
+    return st.value
+
+
+def kivi_stream_decode(shape: dict, params: dict, codes, scales, ring, gauges, *, nthreads: int = 0) -> np.ndarray:
+    """fp64 [L][2][B][H][T][d] of the first T tokens of the stream (t0 = 0)."""
+    sh = dict(t0=0, T_cap=0)
+    sh.update(shape)
+    out = np.zeros(sh["L"] * 2 * sh["B"] * sh["H"] * sh["T"] * sh["d"], np.float64)
+    G = np.ascontiguousarray(gauges, np.float32)
+    rc = lib().cgo_kivi_stream_decode(ctypes.byref(_shape(**sh)), ctypes.byref(_Params(**params)),
+                                      _ptr(np.ascontiguousarray(codes, np.uint8)),
+                                      _ptr(np.ascontiguousarray(scales).view(np.uint16)),
+                                      _ptr(np.ascontiguousarray(ring).view(np.uint16)), _ptr(G), _ptr(out),
+                                      nthreads or (os.cpu_count() or 1))
+    if rc:
+        raise ValueError(f"oracle kivi_stream_decode rc={rc}")
     return out

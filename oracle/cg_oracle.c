@@ -18,7 +18,8 @@
  * Compiled without fast-math and with -ffp-contract=off, so every operation below is
  * the single IEEE operation it reads as.
  *
- * Status of the pins (tests/test_oracle_pins.py, tests/test_oracle_tile_pins.py): every
+ * Status of the pins (tests/test_oracle_pins.py, tests/test_oracle_tile_pins.py,
+ * tests/test_oracle_stream_pins.py): every
  * exported function is pinned against closed forms, brute force, worked examples or
  * library routines; none is "parity unpinned".
  */
@@ -660,3 +661,199 @@ int cgo_decode(const cgo_shape* s, const cgo_params* p, const uint8_t* codes, co
 
 /* The gauge-space value of one coordinate, exposed so that tests can pin the chain. */
 float cgo_gauge_coord(const float* Grow, const float* x, int g) { return gauge_dot(Grow, x, g); }
+
+/* ------------------------------------------------------------------------------ */
+/* KIVI streaming (Sec. 4.3 KIVI-style path; a rolling cache of Sec. 4.4)          */
+/* ------------------------------------------------------------------------------ */
+/* A KIVI history of capacity T_cap tokens per (l, s, b, h) grows by appends. After T tokens
+ * the quantized part holds the first n_q(T) = cgo_kivi_nq(T, R, Gt) tokens, in the batch
+ * layout sized for n_q(T_cap) tokens (quantized groups at fixed places), and the newest
+ * T - n_q(T) tokens stay raw in a ring of W = R + Gt token slots: token t lives in slot
+ * t mod W. The window never holds more than R + Gt - 1 tokens, so no two of its tokens
+ * share a slot. An append of tokens [t0, t0 + T) quantizes every key group that completes,
+ * [n_q(t0), n_q(t0 + T)), reading tokens below t0 from the ring and the others from the new
+ * input, and then stores the new tokens that stay raw. The result equals the batch encode
+ * of all t0 + T tokens (keys and values in the same places, the ring holding the window). */
+
+static int64_t ring_slots(const cgo_params* p) { return (int64_t)p->residual + p->block; }
+
+static int check_stream(const cgo_shape* s, const cgo_params* p)
+{
+    if (!s || !p || p->backend != CGO_KIVI) return CGO_EINVAL;
+    cgo_shape whole = *s;
+    whole.t0 = 0;
+    whole.T = s->T_cap;
+    whole.T_cap = 0;
+    int rc = check_args(&whole, p);
+    if (rc) return rc;
+    if (s->T_cap < 1 || s->t0 < 0 || s->T < 0 || (int64_t)s->t0 + s->T > s->T_cap) return CGO_EINVAL;
+    return CGO_OK;
+}
+
+/* Byte counts of the stream buffers: codes and scales for n_q(T_cap) quantized tokens
+ * (the batch layout at that length), and the ring [L][2][B][H][W][d] of bf16. */
+int cgo_kivi_stream_bytes(const cgo_shape* s, const cgo_params* p, int64_t* codes, int64_t* scales,
+                          int64_t* ring)
+{
+    int rc = check_stream(s, p);
+    if (rc) return rc;
+    cgo_shape cap = *s;
+    cap.t0 = 0;
+    cap.T = s->T_cap;
+    cap.T_cap = 0;
+    int64_t r;
+    cgo_packed_bytes(&cap, p, codes, scales, &r);
+    *ring = (int64_t)s->L * 2 * s->B * s->H * ring_slots(p) * s->d * 2;
+    return CGO_OK;
+}
+
+static const uint16_t* stream_token(const pool_t* P, int64_t unit5, int64_t t)
+{
+    const cgo_shape* s = P->s;
+    int64_t W = ring_slots(P->p);
+    if (t < s->t0) return P->resid + ((size_t)unit5 * W + (size_t)(t % W)) * s->d;
+    return P->x + ((size_t)unit5 * s->T + (size_t)(t - s->t0)) * s->d;
+}
+
+static void kivi_append_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group, Gt = p->block, bits = p->bits, pay = Gt * bits / 8, nb = d / Gt;
+    int64_t R = p->residual, W = ring_slots(p);
+    int64_t nq_old = cgo_kivi_nq(s->t0, R, Gt), nq_new = cgo_kivi_nq((int64_t)s->t0 + s->T, R, Gt);
+    int64_t bh = u % ((int64_t)s->B * s->H), l = u / ((int64_t)s->B * s->H), h = bh % s->H, b = bh / s->H;
+    cgo_shape cap = *s;   /* offsets of the layout sized for the capacity */
+    cap.t0 = 0;
+    cap.T = s->T_cap;
+    cap.T_cap = 0;
+    int64_t kc, vc, ks, vs;
+    kivi_offsets(&cap, p, l, bh, &kc, &vc, &ks, &vs);
+    float* x = (float*)malloc(sizeof(float) * d);
+    float* Z = (float*)malloc(sizeof(float) * (size_t)Gt * d);
+    uint8_t* q = (uint8_t*)malloc((size_t)(Gt > d ? Gt : d));
+    int st = 0;
+    for (int sidx = 0; sidx < 2; sidx++) {
+        int64_t unit5 = ((l * 2 + sidx) * s->B + b) * s->H + h;
+        const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+        if (has_nonfinite(P->x + (size_t)unit5 * s->T * d, (int64_t)s->T * d)) st |= CGO_FLAG_NONFINITE;
+        for (int64_t tg = nq_old / Gt; tg < nq_new / Gt; tg++) {
+            for (int k = 0; k < Gt; k++) {   /* Z of the group's tokens */
+                const uint16_t* xr = stream_token(P, unit5, tg * Gt + k);
+                for (int c = 0; c < d; c++) x[c] = cgo_bf16_to_f32(xr[c]);
+                gauge_apply_f32(Gh, x, Z + (size_t)k * d, d, g);
+            }
+            if (sidx == 0) {   /* keys: per channel over the group */
+                for (int c = 0; c < d; c++) {
+                    uint16_t s16, m16;
+                    st |= quantize_block(Z + c, Gt, d, bits, &s16, &m16, q, NULL, 0);
+                    int64_t idx = tg * d + c;
+                    pack_codes(q, Gt, bits, P->codes + kc + idx * pay);
+                    P->scales[(ks + idx) * 2 + 0] = s16;
+                    P->scales[(ks + idx) * 2 + 1] = m16;
+                }
+            } else {           /* values: per token over blocks of Gt channels */
+                for (int k = 0; k < Gt; k++)
+                    for (int blk = 0; blk < nb; blk++) {
+                        uint16_t s16, m16;
+                        st |= quantize_block(Z + (size_t)k * d + (size_t)blk * Gt, Gt, 1, bits, &s16, &m16, q, NULL, 0);
+                        int64_t idx = (tg * Gt + k) * nb + blk;
+                        pack_codes(q, Gt, bits, P->codes + vc + idx * pay);
+                        P->scales[(vs + idx) * 2 + 0] = s16;
+                        P->scales[(vs + idx) * 2 + 1] = m16;
+                    }
+            }
+        }
+        /* the new tokens that stay raw go to their ring slots (after the reads above) */
+        for (int64_t t = (nq_new > s->t0 ? nq_new : s->t0); t < (int64_t)s->t0 + s->T; t++)
+            memcpy(P->resid + ((size_t)unit5 * W + (size_t)(t % W)) * d,
+                   P->x + ((size_t)unit5 * s->T + (size_t)(t - s->t0)) * d, sizeof(uint16_t) * d);
+    }
+    add_status(P, st);
+    free(x);
+    free(Z);
+    free(q);
+}
+
+/* Append tokens [t0, t0 + T) (x_new: bf16 [L][2][B][H][T][d]) to a KIVI stream of capacity
+ * T_cap that holds t0 tokens: codes, scales and ring as laid out above. */
+int cgo_kivi_append(const cgo_shape* s, const cgo_params* p, const uint16_t* x_new, const float* G, uint8_t* codes,
+                    uint16_t* scales, uint16_t* ring, int nthreads, int32_t* status_out)
+{
+    int rc = check_stream(s, p);
+    if (rc) return rc;
+    pool_t P;
+    memset(&P, 0, sizeof P);
+    P.s = s; P.p = p; P.x = x_new; P.G = G; P.codes = codes; P.scales = scales; P.resid = ring;
+    P.n_units = (int64_t)s->L * s->B * s->H;
+    P.fn = kivi_append_unit;
+    run_pool(&P, nthreads);
+    if (status_out) *status_out = P.status;
+    return CGO_OK;
+}
+
+static void kivi_stream_decode_unit(void* ctx, int64_t u)
+{
+    pool_t* P = (pool_t*)ctx;
+    const cgo_shape* s = P->s;
+    const cgo_params* p = P->p;
+    int d = s->d, g = p->group, Gt = p->block, bits = p->bits, pay = Gt * bits / 8, nb = d / Gt;
+    int64_t W = ring_slots(p), T = s->T, nq = cgo_kivi_nq(T, p->residual, Gt);
+    int64_t bh = u % ((int64_t)s->B * s->H), l = u / ((int64_t)s->B * s->H), h = bh % s->H, b = bh / s->H;
+    cgo_shape cap = *s;
+    cap.t0 = 0;
+    cap.T = s->T_cap;
+    cap.T_cap = 0;
+    int64_t kc, vc, ks, vs;
+    kivi_offsets(&cap, p, l, bh, &kc, &vc, &ks, &vs);
+    double* zh = (double*)malloc(sizeof(double) * d);
+    uint8_t* q = (uint8_t*)malloc((size_t)(Gt > d ? Gt : d));
+    for (int sidx = 0; sidx < 2; sidx++) {
+        int64_t unit5 = ((l * 2 + sidx) * s->B + b) * s->H + h;
+        const float* Gh = P->G + ((size_t)(l * 2 + sidx) * s->H + h) * (size_t)d * g;
+        double* out = P->xhat + (size_t)unit5 * T * d;
+        for (int64_t t = 0; t < nq; t++) {
+            for (int c = 0; c < d; c++) {   /* zhat of token t */
+                int64_t idx, k;
+                uint16_t sc16, mz16;
+                if (sidx == 0) {
+                    idx = (t / Gt) * d + c;
+                    k = t % Gt;
+                    unpack_codes(P->in_codes + kc + idx * pay, Gt, bits, q);
+                    sc16 = P->in_scales[(ks + idx) * 2 + 0];
+                    mz16 = P->in_scales[(ks + idx) * 2 + 1];
+                } else {
+                    idx = t * nb + c / Gt;
+                    k = c % Gt;
+                    unpack_codes(P->in_codes + vc + idx * pay, Gt, bits, q);
+                    sc16 = P->in_scales[(vs + idx) * 2 + 0];
+                    mz16 = P->in_scales[(vs + idx) * 2 + 1];
+                }
+                zh[c] = (double)q[k] * (double)cgo_f16_to_f32(sc16) + (double)cgo_f16_to_f32(mz16);
+            }
+            gauge_inverse_f64(Gh, zh, out + (size_t)t * d, d, g);
+        }
+        for (int64_t t = nq; t < T; t++)
+            for (int c = 0; c < d; c++)
+                out[(size_t)t * d + c] = (double)cgo_bf16_to_f32(P->in_resid[((size_t)unit5 * W + (size_t)(t % W)) * d + c]);
+    }
+    free(zh);
+    free(q);
+}
+
+/* Decode the first T tokens of a KIVI stream (t0 must be 0): xhat fp64 [L][2][B][H][T][d]. */
+int cgo_kivi_stream_decode(const cgo_shape* s, const cgo_params* p, const uint8_t* codes, const uint16_t* scales,
+                           const uint16_t* ring, const float* G, double* xhat, int nthreads)
+{
+    int rc = check_stream(s, p);
+    if (rc) return rc;
+    if (s->t0 != 0) return CGO_EUNSUP;
+    pool_t P;
+    memset(&P, 0, sizeof P);
+    P.s = s; P.p = p; P.G = G; P.in_codes = codes; P.in_scales = scales; P.in_resid = ring; P.xhat = xhat;
+    P.n_units = (int64_t)s->L * s->B * s->H;
+    P.fn = kivi_stream_decode_unit;
+    run_pool(&P, nthreads);
+    return CGO_OK;
+}

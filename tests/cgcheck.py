@@ -195,3 +195,28 @@ def compare_decode(w, got_bf16: np.ndarray, ref: np.ndarray, G: np.ndarray, step
         tol_rel = decode_tolerance(w, ref, G, step_mism, rms_floor=False).reshape(-1)
         stats["rms_floor_only"] = int((loose & (err > tol_rel)).sum())
     return stats
+
+
+def stream_to_batch(w, T: int, T_cap: int, codes: np.ndarray, scales_u16: np.ndarray, ring_u16: np.ndarray):
+    """The state of a KIVI stream of capacity T_cap holding T tokens, in the batch layout of a
+    T-token KIVI encode: (codes, scales, residual). Keys [B][H][n_q/Gt][d][pay] and values
+    [B][H][n_q][d/Gt][pay] per layer are cut from the capacity layout; the residual tokens
+    [n_q, T) come from ring slot t mod (R + Gt)."""
+    L, B, H, d, Gt, bits, R = w.L, w.B, w.H, w.d, w.block, w.bits, w.residual
+    pay, nb, W = Gt * bits // 8, d // Gt, R + Gt
+    nq, ncap = oracle.kivi_nq(T, R, Gt), oracle.kivi_nq(T_cap, R, Gt)
+    kc_cap, vc_cap = (ncap // Gt) * d * pay, ncap * nb * pay
+    ks_cap, vs_cap = (ncap // Gt) * d, ncap * nb
+    c = codes.reshape(L, -1)
+    s = scales_u16.reshape(-1, 2).reshape(L, -1, 2)
+    out_c, out_s = [], []
+    for l in range(L):
+        kc = c[l, :B * H * kc_cap].reshape(B, H, kc_cap)[:, :, :(nq // Gt) * d * pay]
+        vc = c[l, B * H * kc_cap:].reshape(B, H, vc_cap)[:, :, :nq * nb * pay]
+        ks = s[l, :B * H * ks_cap].reshape(B, H, ks_cap, 2)[:, :, :(nq // Gt) * d]
+        vs = s[l, B * H * ks_cap:].reshape(B, H, vs_cap, 2)[:, :, :nq * nb]
+        out_c += [kc.ravel(), vc.ravel()]
+        out_s += [ks.ravel(), vs.ravel()]
+    ring = ring_u16.reshape(L, 2, B, H, W, d)
+    resid = ring[:, :, :, :, np.arange(nq, T) % W, :]
+    return np.concatenate(out_c), np.concatenate(out_s), np.ascontiguousarray(resid).ravel()
