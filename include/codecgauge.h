@@ -146,6 +146,45 @@ int cg_decode(const cg_shape* shape, const cg_params* params,
               const void* codes, const void* scales, const void* residual,
               const float* gauges, void* out_kv_bf16, void* stream);
 
+/* ---- KIVI streaming (Sec. 4.3 KIVI-style path; the growing cache of a decode loop) ----
+ * A KIVI history of capacity T_cap tokens per (l, s, b, h) that grows by appends. Holding
+ * T tokens, its first n_q(T) = max(0, floor((T - residual) / block)) * block tokens are
+ * quantized and the newest T - n_q(T) stay raw (KIVI's full-precision window). Buffers:
+ *   codes, scales : the CG_KIVI layouts above, sized for n_q(T_cap) quantized tokens
+ *                   (a layer's keys for n_q(T_cap)/block groups, then its values); group k
+ *                   and token t sit at the same place whatever T is
+ *   ring          : bf16 [L][2][B][H][W][d], W = residual + block; raw token t lives in
+ *                   slot t mod W (the window never holds more than W - 1 tokens)
+ *   workspace     : device scratch of cg_kivi_stream_bytes' workspace size, owned by the
+ *                   caller; an append that completes a key group stages the group's tokens
+ *                   (ring and new input) there before quantizing them
+ * The stream state after any sequence of appends equals the CG_KIVI encode of all tokens so
+ * far (same codes and scales; the ring holds the raw window). */
+
+/* Byte counts of the stream buffers for capacity shape->T_cap (shape->t0 and T must satisfy
+ * t0 + T <= T_cap; they do not change the counts): codes, scales, ring, and the workspace an
+ * append with t0 > 0 needs (L*2*B*H*block*d*2; 0 would do for appends that start at 0).
+ * Host-only. CG_EINVAL on invalid arguments (backend must be CG_KIVI, T_cap >= 1). */
+int cg_kivi_stream_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes,
+                         size_t* scales_bytes, size_t* ring_bytes, size_t* workspace_bytes);
+
+/* Append tokens [t0, t0 + T) to a stream that holds t0 tokens. kv_new: bf16 [L][2][B][H][T][d]
+ * (the new tokens only). t0 = 0 starts the stream (a prefill of any length); after that an
+ * append carries at most `block` tokens (CG_EUNSUPPORTED otherwise), so it completes at most
+ * one key group. workspace may be NULL when t0 = 0; otherwise it must hold the workspace size
+ * (CG_EINVAL if workspace_bytes is smaller). Launches up to four kernels in order on
+ * `stream` (stage, keys, values, ring); a CG_ECUDA may follow queued launches, and the
+ * stream state is then invalid. Pointers 16-byte aligned. */
+int cg_kivi_append(const cg_shape* shape, const cg_params* params, const void* kv_new_bf16,
+                   const float* gauges, void* codes, void* scales, void* ring, void* workspace,
+                   size_t workspace_bytes, void* stream);
+
+/* Decode the T tokens a stream holds (shape->t0 must be 0, T <= T_cap): quantized tokens as
+ * cg_decode does, raw tokens copied from the ring, into out_kv_bf16 [L][2][B][H][T][d]. */
+int cg_kivi_stream_decode(const cg_shape* shape, const cg_params* params, const void* codes,
+                          const void* scales, const void* ring, const float* gauges,
+                          void* out_kv_bf16, void* stream);
+
 /* Reads and clears (in one atomic step, ordered on `stream`) the accumulated CG_FLAG_* bits
  * of the current device, synchronizes `stream` and returns them in *device_flags. Returns
  * CG_ECUDA if a launch, copy or the synchronize fails. The limit of each bounded pipeline

@@ -17,7 +17,8 @@ import os
 from dataclasses import dataclass
 
 __all__ = ["CG_BLOCK_UNIFORM", "CG_KIVI", "CG_NONE", "CG_BLOCK_TILE", "CG_TILE_TOKENS", "Shape", "Params",
-           "packed_bytes", "encode", "decode", "get_status", "lib_path", "load", "CodecGaugeError"]
+           "packed_bytes", "encode", "decode", "get_status", "lib_path", "load", "CodecGaugeError",
+           "kivi_stream_bytes", "kivi_stream_alloc", "kivi_append", "kivi_stream_decode"]
 
 CG_BLOCK_UNIFORM, CG_KIVI, CG_NONE, CG_BLOCK_TILE = 0, 1, 2, 3
 CG_TILE_TOKENS = 16
@@ -90,6 +91,12 @@ def load():
         L.cg_encode.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp]
         L.cg_decode.restype = ctypes.c_int
         L.cg_decode.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp]
+        L.cg_kivi_stream_bytes.restype = ctypes.c_int
+        L.cg_kivi_stream_bytes.argtypes = [P(_CShape), P(_CParams)] + [P(ctypes.c_size_t)] * 4
+        L.cg_kivi_append.restype = ctypes.c_int
+        L.cg_kivi_append.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+        L.cg_kivi_stream_decode.restype = ctypes.c_int
+        L.cg_kivi_stream_decode.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp]
         L.cg_get_status.restype = ctypes.c_int
         L.cg_get_status.argtypes = [vp, P(ctypes.c_int32)]
         L.cg_last_error.restype = ctypes.c_char_p
@@ -131,6 +138,39 @@ def decode(shape: Shape, params: Params, codes, scales, residual, gauges, out, s
     """Decode (Zhat = D(B_c), Xhat = G^T Zhat) into the caller's bf16 output tensor."""
     _check(load().cg_decode(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(codes), _ptr(scales),
                             _ptr(residual), _ptr(gauges), _ptr(out), _stream(stream)))
+
+
+def kivi_stream_bytes(shape: Shape, params: Params) -> tuple[int, int, int, int]:
+    """(codes, scales, ring, workspace) byte counts of a KIVI stream of capacity shape.T_cap."""
+    v = [ctypes.c_size_t() for _ in range(4)]
+    _check(load().cg_kivi_stream_bytes(ctypes.byref(shape.c()), ctypes.byref(params.c()),
+                                       *[ctypes.byref(x) for x in v]))
+    return tuple(x.value for x in v)
+
+
+def kivi_stream_alloc(shape: Shape, params: Params, device="cuda"):
+    """Zero-filled device buffers (codes, scales, ring, workspace) of a KIVI stream."""
+    import torch
+    nc, ns, nr, nw = kivi_stream_bytes(shape, params)
+    return (torch.zeros(max(nc, 16), dtype=torch.uint8, device=device),
+            torch.zeros(max(ns // 4, 4), dtype=torch.int32, device=device),
+            torch.zeros(max(nr // 2, 8), dtype=torch.int16, device=device),
+            torch.zeros(max(nw // 2, 8), dtype=torch.int16, device=device))
+
+
+def kivi_append(shape: Shape, params: Params, kv_new, gauges, codes, scales, ring, workspace=None,
+                stream=None) -> None:
+    """Append tokens [t0, t0 + T) (kv_new holds only them) to a KIVI stream holding t0 tokens."""
+    nbytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _check(load().cg_kivi_append(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(kv_new), _ptr(gauges),
+                                 _ptr(codes), _ptr(scales), _ptr(ring), _ptr(workspace), nbytes,
+                                 _stream(stream)))
+
+
+def kivi_stream_decode(shape: Shape, params: Params, codes, scales, ring, gauges, out, stream=None) -> None:
+    """Decode the T tokens a KIVI stream holds (shape.t0 = 0) into the caller's bf16 output."""
+    _check(load().cg_kivi_stream_decode(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(codes),
+                                        _ptr(scales), _ptr(ring), _ptr(gauges), _ptr(out), _stream(stream)))
 
 
 def get_status(stream=None) -> int:

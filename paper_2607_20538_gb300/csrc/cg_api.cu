@@ -271,6 +271,131 @@ KeyArgs key_args(const cg_shape* sh, const cg_params* p, const Sizes& z, int32_t
     return k;
 }
 
+// KIVI quantized part, encode: the t_count tokens (whole key groups) in rows [0, t_count) of
+// x [L][2][B][H][T_x][d] become quantized tokens [tok0, tok0 + t_count) of the layout z (tok0 a
+// multiple of the group length). Keys on tensor cores where eligible, else on CUDA cores;
+// values through the row kernels. Sets *what to the failing launch.
+cudaError_t kivi_encode_groups(const cg_shape* sh, const cg_params* p, const Sizes& z, const uint16_t* x,
+                               int64_t T_x, int64_t t_count, int64_t tok0, const float* G, uint8_t* codes,
+                               uint32_t* scales, int32_t* status, cudaStream_t st, const char** what) {
+    const int64_t Gt = p->block, gi = tok0 / Gt;
+    RowArgs a = row_args(sh, p, status);
+    a.x = x;
+    a.G = G;
+    a.codes = codes;
+    a.scales = scales;
+    a.T_x = T_x;
+    a.t_count = t_count;
+    RowArgs ka = a;  // keys: s = 0, one block per channel and key group
+    ka.s_lo = 0;
+    ka.s_n = 1;
+    kivi_key_maps(sh, p, z, &ka.cmap, &ka.smap);
+    ka.cmap.base += gi * sh->d * z.pay;
+    ka.smap.base += gi * sh->d;
+    cudaError_t e;
+    if (tc_key_encode_eligible(ka)) {
+        e = tc_launch_key_encode(ka, st);
+    } else {
+        KeyArgs k = key_args(sh, p, z, status);
+        k.x = x;
+        k.T = T_x;
+        k.nq = t_count;
+        k.G = G;
+        k.codes = codes + gi * sh->d * z.pay;
+        k.scales = scales + gi * sh->d;
+        e = launch_key_encode_simt(k, st);
+    }
+    if (e != cudaSuccess) {
+        *what = "KIVI key encode launch";
+        return e;
+    }
+    a.s_lo = 1;
+    a.s_n = 1;
+    kivi_value_maps(sh, z, &a.cmap, &a.smap);
+    a.cmap.base += tok0 * z.nb * z.pay;
+    a.smap.base += tok0 * z.nb;
+    e = tc_row_encode_eligible(a) ? tc_launch_row_encode(a, st) : launch_row_encode_simt(a, st);
+    if (e != cudaSuccess) *what = "KIVI value encode launch";
+    return e;
+}
+
+// KIVI quantized part, decode: quantized tokens [0, t_count) of the layout z into rows
+// [0, t_count) of out [L][2][B][H][T_x][d].
+cudaError_t kivi_decode_groups(const cg_shape* sh, const cg_params* p, const Sizes& z, const uint8_t* codes,
+                               const uint32_t* scales, const float* G, uint16_t* out, int64_t T_x, int64_t t_count,
+                               int32_t* status, cudaStream_t st, const char** what) {
+    RowArgs a = row_args(sh, p, status);
+    a.out = out;
+    a.G = G;
+    a.codes = const_cast<uint8_t*>(codes);
+    a.scales = const_cast<uint32_t*>(scales);
+    a.T_x = T_x;
+    a.t_count = t_count;
+    RowArgs ka = a;  // keys: s = 0, one 128-token group per tile
+    ka.s_lo = 0;
+    ka.s_n = 1;
+    kivi_key_maps(sh, p, z, &ka.cmap, &ka.smap);
+    cudaError_t e;
+    if (tc_key_decode_eligible(ka)) {
+        e = tc_launch_key_decode(ka, st);
+    } else {
+        KeyArgs k = key_args(sh, p, z, status);
+        k.out = out;
+        k.T = T_x;
+        k.nq = t_count;
+        k.G = G;
+        k.codes = a.codes;
+        k.scales = a.scales;
+        e = launch_key_decode_simt(k, st);
+    }
+    if (e != cudaSuccess) {
+        *what = "KIVI key decode launch";
+        return e;
+    }
+    a.s_lo = 1;
+    a.s_n = 1;
+    kivi_value_maps(sh, z, &a.cmap, &a.smap);
+    e = tc_row_decode_eligible(a) ? tc_launch_row_decode(a, st) : launch_row_decode_simt(a, st);
+    if (e != cudaSuccess) *what = "KIVI value decode launch";
+    return e;
+}
+
+// Sizes of a KIVI stream of capacity sh->T_cap: the CG_KIVI layout at T_cap tokens, the ring
+// of W = residual + block slots and the staging workspace of one key group per unit.
+struct StreamSizes {
+    Sizes z;
+    int64_t W;
+    size_t ring, workspace;
+};
+
+int validate_stream(const cg_shape* sh, const cg_params* p, StreamSizes* ss) {
+    if (!sh || !p) return fail(CG_EINVAL, "null shape or params");
+    if (p->backend != CG_KIVI) return fail(CG_EINVAL, "KIVI streaming needs backend CG_KIVI");
+    if (sh->T_cap < 1 || sh->t0 < 0 || sh->T < 0 || (int64_t)sh->t0 + sh->T > sh->T_cap)
+        return fail(CG_EINVAL, "KIVI stream: needs T_cap >= 1 and 0 <= t0, t0 + T <= T_cap (t0=%d T=%d T_cap=%d)",
+                    sh->t0, sh->T, sh->T_cap);
+    cg_shape cap = *sh;
+    cap.t0 = 0;
+    cap.T = sh->T_cap;
+    cap.T_cap = 0;
+    int rc = validate(&cap, p, &ss->z);
+    if (rc) return rc;
+    ss->W = (int64_t)p->residual + p->block;
+    const size_t units = (size_t)sh->L * 2 * sh->B * sh->H;
+    size_t row = (size_t)sh->d * 2;
+    if (!mul_ok(units * row, (size_t)ss->W, &ss->ring)) return fail(CG_ERANGE, "size overflow");
+    if (!mul_ok(units * row, (size_t)p->block, &ss->workspace)) return fail(CG_ERANGE, "size overflow");
+    return CG_OK;
+}
+
+MoveArgs move_args(const cg_shape* sh, int64_t W) {
+    MoveArgs m{};
+    m.units = (int64_t)sh->L * 2 * sh->B * sh->H;
+    m.d = sh->d;
+    m.W = W;
+    return m;
+}
+
 }  // namespace
 }  // namespace cg
 
@@ -334,28 +459,9 @@ CG_EXPORT int cg_encode(const cg_shape* shape, const cg_params* params, const vo
         return CG_OK;
     }
     if (z.nq > 0) {
-        RowArgs ka = a;  // keys on tensor cores: s = 0, one block per channel and key group
-        ka.s_lo = 0;
-        ka.s_n = 1;
-        ka.t_count = z.nq;
-        kivi_key_maps(shape, params, z, &ka.cmap, &ka.smap);
-        if (tc_key_encode_eligible(ka)) {
-            e = tc_launch_key_encode(ka, st);
-        } else {
-            KeyArgs k = key_args(shape, params, z, status);
-            k.x = a.x;
-            k.G = gauges;
-            k.codes = a.codes;
-            k.scales = a.scales;
-            e = launch_key_encode_simt(k, st);
-        }
-        if (e != cudaSuccess) return cuda_fail(e, "KIVI key encode launch");
-        a.s_lo = 1;
-        a.s_n = 1;
-        a.t_count = z.nq;
-        kivi_value_maps(shape, z, &a.cmap, &a.smap);
-        e = tc_row_encode_eligible(a) ? tc_launch_row_encode(a, st) : launch_row_encode_simt(a, st);
-        if (e != cudaSuccess) return cuda_fail(e, "KIVI value encode launch");
+        const char* what = "";
+        e = kivi_encode_groups(shape, params, z, a.x, shape->T, z.nq, 0, gauges, a.codes, a.scales, status, st, &what);
+        if (e != cudaSuccess) return cuda_fail(e, what);
     }
     if (shape->T - z.nq > 0) {
         ResidArgs r{};
@@ -408,28 +514,9 @@ CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const vo
         return CG_OK;
     }
     if (z.nq > 0) {
-        RowArgs ka = a;  // keys on tensor cores: s = 0, one 128-token group per tile
-        ka.s_lo = 0;
-        ka.s_n = 1;
-        ka.t_count = z.nq;
-        kivi_key_maps(shape, params, z, &ka.cmap, &ka.smap);
-        if (tc_key_decode_eligible(ka)) {
-            e = tc_launch_key_decode(ka, st);
-        } else {
-            KeyArgs k = key_args(shape, params, z, status);
-            k.out = a.out;
-            k.G = gauges;
-            k.codes = a.codes;
-            k.scales = a.scales;
-            e = launch_key_decode_simt(k, st);
-        }
-        if (e != cudaSuccess) return cuda_fail(e, "KIVI key decode launch");
-        a.s_lo = 1;
-        a.s_n = 1;
-        a.t_count = z.nq;
-        kivi_value_maps(shape, z, &a.cmap, &a.smap);
-        e = tc_row_decode_eligible(a) ? tc_launch_row_decode(a, st) : launch_row_decode_simt(a, st);
-        if (e != cudaSuccess) return cuda_fail(e, "KIVI value decode launch");
+        const char* what = "";
+        e = kivi_decode_groups(shape, params, z, a.codes, a.scales, gauges, a.out, shape->T, z.nq, status, st, &what);
+        if (e != cudaSuccess) return cuda_fail(e, what);
     }
     if (shape->T - z.nq > 0) {
         ResidArgs r{};
@@ -443,6 +530,124 @@ CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const vo
         e = launch_residual_copy(r, st);
         if (e != cudaSuccess) return cuda_fail(e, "KIVI residual copy launch");
     }
+    return CG_OK;
+}
+
+CG_EXPORT int cg_kivi_stream_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes,
+                                   size_t* scales_bytes, size_t* ring_bytes, size_t* workspace_bytes) {
+    t_err.clear();
+    StreamSizes ss;
+    int rc = validate_stream(shape, params, &ss);
+    if (rc) return rc;
+    if (codes_bytes) *codes_bytes = ss.z.codes;
+    if (scales_bytes) *scales_bytes = ss.z.scales;
+    if (ring_bytes) *ring_bytes = ss.ring;
+    if (workspace_bytes) *workspace_bytes = ss.workspace;
+    return CG_OK;
+}
+
+CG_EXPORT int cg_kivi_append(const cg_shape* shape, const cg_params* params, const void* kv_new_bf16,
+                             const float* gauges, void* codes, void* scales, void* ring, void* workspace,
+                             size_t workspace_bytes, void* stream) {
+    t_err.clear();
+    StreamSizes ss;
+    int rc = validate_stream(shape, params, &ss);
+    if (rc) return rc;
+    const int64_t t0 = shape->t0, T = shape->T, Gt = params->block, R = params->residual;
+    if (t0 > 0 && T > Gt)
+        return fail(CG_EUNSUPPORTED, "KIVI stream: an append after the first call carries at most block=%d tokens "
+                    "(got T=%d)", params->block, shape->T);
+    if (T == 0) return CG_OK;
+    const int64_t nq_old = kivi_nq(t0, R, Gt), nq_new = kivi_nq(t0 + T, R, Gt);
+    const bool stage = t0 > 0 && nq_new > nq_old;
+    if (!kv_new_bf16 || !gauges || !ring) return fail(CG_EINVAL, "null kv, gauges or ring pointer");
+    if (nq_new > nq_old && (!codes || !scales)) return fail(CG_EINVAL, "null codes or scales");
+    if (stage && (!workspace || workspace_bytes < ss.workspace))
+        return fail(CG_EINVAL, "this append completes a key group: workspace needs %zu bytes (got %zu)", ss.workspace,
+                    workspace ? workspace_bytes : (size_t)0);
+    if (!aligned16(kv_new_bf16) || !aligned16(gauges) || !aligned16(codes) || !aligned16(scales) ||
+        !aligned16(ring) || !aligned16(workspace))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const uint16_t* x = static_cast<const uint16_t*>(kv_new_bf16);
+    uint16_t* rg = static_cast<uint16_t*>(ring);
+    cudaError_t e = cudaSuccess;
+    const char* what = "";
+    if (nq_new > nq_old) {
+        if (stage) {
+            // the completed group's tokens, from the ring (t < t0) and the new input, staged
+            // as a dense [L][2][B][H][block][d] input
+            MoveArgs m = move_args(shape, ss.W);
+            m.ring_src = rg;
+            m.x = x;
+            m.T_x = T;
+            m.x_t0 = t0;
+            m.src_split = t0;
+            m.t_lo = nq_old;
+            m.t_hi = nq_new;
+            m.dst = static_cast<uint16_t*>(workspace);
+            m.dst_T = Gt;
+            m.dst_t0 = nq_old;
+            if ((e = launch_row_move(m, st)) != cudaSuccess) return cuda_fail(e, "KIVI stream staging launch");
+            e = kivi_encode_groups(shape, params, ss.z, static_cast<const uint16_t*>(workspace), Gt, Gt, nq_old,
+                                   gauges, static_cast<uint8_t*>(codes), static_cast<uint32_t*>(scales), status, st,
+                                   &what);
+        } else {
+            e = kivi_encode_groups(shape, params, ss.z, x, T, nq_new, 0, gauges, static_cast<uint8_t*>(codes),
+                                   static_cast<uint32_t*>(scales), status, st, &what);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, what);
+    }
+    // new tokens that stay raw go to their ring slots (after the staging read above)
+    MoveArgs m = move_args(shape, ss.W);
+    m.x = x;
+    m.T_x = T;
+    m.x_t0 = t0;
+    m.src_split = 0;
+    m.t_lo = nq_new > t0 ? nq_new : t0;
+    m.t_hi = t0 + T;
+    m.dst = rg;
+    m.dst_ring = 1;
+    if ((e = launch_row_move(m, st)) != cudaSuccess) return cuda_fail(e, "KIVI stream ring launch");
+    return CG_OK;
+}
+
+CG_EXPORT int cg_kivi_stream_decode(const cg_shape* shape, const cg_params* params, const void* codes,
+                                    const void* scales, const void* ring, const float* gauges, void* out_kv_bf16,
+                                    void* stream) {
+    t_err.clear();
+    StreamSizes ss;
+    int rc = validate_stream(shape, params, &ss);
+    if (rc) return rc;
+    if (shape->t0 != 0) return fail(CG_EUNSUPPORTED, "KIVI stream decode reads the whole history: t0 must be 0");
+    const int64_t T = shape->T, nq = kivi_nq(T, params->residual, params->block);
+    if (T == 0) return CG_OK;
+    if (!out_kv_bf16 || !gauges || !ring) return fail(CG_EINVAL, "null output, gauges or ring pointer");
+    if (nq > 0 && (!codes || !scales)) return fail(CG_EINVAL, "null codes or scales");
+    if (!aligned16(codes) || !aligned16(scales) || !aligned16(ring) || !aligned16(gauges) || !aligned16(out_kv_bf16))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint16_t* out = static_cast<uint16_t*>(out_kv_bf16);
+    cudaError_t e = cudaSuccess;
+    if (nq > 0) {
+        const char* what = "";
+        e = kivi_decode_groups(shape, params, ss.z, static_cast<const uint8_t*>(codes),
+                               static_cast<const uint32_t*>(scales), gauges, out, T, nq, status, st, &what);
+        if (e != cudaSuccess) return cuda_fail(e, what);
+    }
+    MoveArgs m = move_args(shape, ss.W);
+    m.ring_src = static_cast<const uint16_t*>(ring);
+    m.src_split = T;  // every raw token comes from the ring
+    m.t_lo = nq;
+    m.t_hi = T;
+    m.dst = out;
+    m.dst_T = T;
+    m.dst_t0 = 0;
+    if ((e = launch_row_move(m, st)) != cudaSuccess) return cuda_fail(e, "KIVI stream window launch");
     return CG_OK;
 }
 

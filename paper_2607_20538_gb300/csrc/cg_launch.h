@@ -50,7 +50,23 @@ struct ResidArgs {
     int to_residual;        // 1: x -> residual window, 0: residual window -> out
 };
 
+// Token-row moves of the KIVI stream: rows t in [t_lo, t_hi) of every (l, s, b, h) unit.
+// Source row t: ring slot t mod W when t < src_split, else row t - x_t0 of the dense x
+// ([units][T_x][d]). Destination: ring slot t mod W (dst_ring) or dense row t - dst_t0 of
+// [units][dst_T][d].
+struct MoveArgs {
+    const uint16_t* ring_src;
+    const uint16_t* x;
+    uint16_t* dst;
+    int64_t units, d, W;
+    int64_t T_x, x_t0, src_split;
+    int64_t t_lo, t_hi;
+    int dst_ring;
+    int64_t dst_T, dst_t0;
+};
+
 cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st);
+cudaError_t launch_row_move(const MoveArgs& a, cudaStream_t st);
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st);

@@ -572,7 +572,30 @@ __global__ void residual_copy_kernel(ResidArgs a) {
     }
 }
 
+__global__ void __launch_bounds__(256) row_move_kernel(MoveArgs a) {
+    const int64_t c16 = a.d / 8;  // 16-byte chunks per token row
+    const int64_t rows = a.t_hi - a.t_lo;
+    const int64_t n = a.units * rows * c16;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t u = i / (rows * c16), rem = i - u * rows * c16;
+        const int64_t t = a.t_lo + rem / c16, c = rem % c16;
+        const uint16_t* src = t < a.src_split ? a.ring_src + (u * a.W + t % a.W) * a.d
+                                              : a.x + (u * a.T_x + (t - a.x_t0)) * a.d;
+        uint16_t* dst = a.dst_ring ? a.dst + (u * a.W + t % a.W) * a.d : a.dst + (u * a.dst_T + (t - a.dst_t0)) * a.d;
+        reinterpret_cast<uint4*>(dst)[c] = reinterpret_cast<const uint4*>(src)[c];
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_row_move(const MoveArgs& a, cudaStream_t st) {
+    const int64_t n = a.units * (a.t_hi - a.t_lo) * (a.d / 8);
+    if (n <= 0) return cudaSuccess;
+    int64_t blocks = (n + 255) / 256;
+    if (blocks > 152 * 16) blocks = 152 * 16;
+    row_move_kernel<<<(unsigned)blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
 
 // Warps per CTA of the tile encode kernel: as many as shared memory holds, at most 16.
 static int tile_simt_warps(int d, int g) {

@@ -85,6 +85,28 @@ def test_tile_history_offsets(lib):
             assert e.value.code == (-1 if t0 + T > T_cap else -2)
 
 
+def test_kivi_stream_bytes_and_validation(lib):
+    """Stream byte counts as the oracle counts them; argument errors before any device work."""
+    params = cg.Params(cg.CG_KIVI, 16, 3, 16, 20)
+    for T_cap in (1, 20, 36, 37, 300):
+        sh = dict(L=2, B=2, H=3, T=0, d=64, t0=0, T_cap=T_cap)
+        nc, ns, nr, nw = cg.kivi_stream_bytes(cg.Shape(**sh), params)
+        assert (nc, ns, nr) == oracle.kivi_stream_bytes(sh, params.__dict__)
+        assert nw == 2 * 2 * 2 * 3 * 16 * 64 * 2
+    S = lambda **k: ctypes.byref(cg.Shape(**{**dict(L=1, B=1, H=1, T=1, d=64, t0=0, T_cap=64), **k}).c())
+    P = ctypes.byref(params.c())
+    fake = ctypes.c_void_p(0x10000)
+    assert lib.cg_kivi_stream_bytes(S(T_cap=0), P, None, None, None, None) == -1
+    assert lib.cg_kivi_stream_bytes(S(t0=60, T=5), P, None, None, None, None) == -1
+    assert lib.cg_kivi_stream_bytes(S(), ctypes.byref(cg.Params(0, 16, 3, 16).c()), None, None, None, None) == -1
+    # appends after the first call carry at most `block` tokens
+    assert lib.cg_kivi_append(S(t0=4, T=17), P, fake, fake, fake, fake, fake, fake, 1 << 20, None) == -2
+    # an append that completes a key group (t0 = 35 -> 36 tokens: n_q 0 -> 16) needs the workspace
+    assert lib.cg_kivi_append(S(t0=35, T=1), P, fake, fake, fake, fake, fake, fake, 16, None) == -1
+    assert "workspace" in lib.cg_last_error().decode()
+    assert lib.cg_kivi_stream_decode(S(t0=1, T=2), P, fake, fake, fake, fake, fake, None) == -2
+
+
 def test_pointer_checks_fail_before_device(lib):
     shape = cg.Shape(L=1, B=1, H=1, T=4, d=64)
     params = cg.Params(0, 16, 4, 32)
