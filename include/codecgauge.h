@@ -179,6 +179,22 @@ int cg_kivi_append(const cg_shape* shape, const cg_params* params, const void* k
                    const float* gauges, void* codes, void* scales, void* ring, void* workspace,
                    size_t workspace_bytes, void* stream);
 
+/* Bytes of the library's own workspace array used by cg_kivi_append_static. */
+#define CG_KIVI_APPEND_STATIC_BYTES (32u * 1024u * 1024u)
+
+/* cg_kivi_append without a caller-allocated workspace. The paper has no counterpart: this is
+ * an interface for callers that cannot allocate device memory (a framework's memory pool with
+ * no hook for extra buffers, memory reserved up front, a real-time loop where an allocation
+ * could block or fail). The staging workspace is a fixed array of CG_KIVI_APPEND_STATIC_BYTES
+ * in the library's device memory; the call allocates and frees nothing. Arguments and results
+ * are those of cg_kivi_append. Shapes whose workspace size (cg_kivi_stream_bytes) exceeds the
+ * array return CG_ERANGE whatever t0 is (call per layer instead). The first call on each
+ * device looks up the array's address with that device current: make it before any stream
+ * capture. All calls share the array, so calls whose kernels overlap on the GPU race on it.
+ * Nothing in it needs to start at zero. */
+int cg_kivi_append_static(const cg_shape* shape, const cg_params* params, const void* kv_new_bf16,
+                          const float* gauges, void* codes, void* scales, void* ring, void* stream);
+
 /* Decode the T tokens a stream holds (shape->t0 must be 0, T <= T_cap): quantized tokens as
  * cg_decode does, raw tokens copied from the ring, into out_kv_bf16 [L][2][B][H][T][d]. */
 int cg_kivi_stream_decode(const cg_shape* shape, const cg_params* params, const void* codes,

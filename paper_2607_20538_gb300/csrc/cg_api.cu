@@ -397,6 +397,17 @@ MoveArgs move_args(const cg_shape* sh, int64_t W) {
 }
 
 }  // namespace
+
+int set_error(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    t_err = buf;
+    return code;
+}
+
 }  // namespace cg
 
 using namespace cg;

@@ -65,6 +65,9 @@ struct MoveArgs {
     int64_t dst_T, dst_t0;
 };
 
+// Sets the message cg_last_error() returns on this host thread; returns code.
+int set_error(int code, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+
 cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_row_move(const MoveArgs& a, cudaStream_t st);
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st);
