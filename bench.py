@@ -368,6 +368,82 @@ def _setup_rolling(w, dev, ws, stream):
     return P
 
 
+def _setup_kivi_stream(w, dev, ws, stream):
+    """KIVI decode-loop step over a stream of capacity T_cap holding T_cap - 1 tokens: append one
+    token per sequence at T_cap - 1 (it completes a key group, so the step also stages and
+    quantizes that group's 128 keys and values), then decode all T_cap tokens. The history is
+    prefilled once before timing, layer by layer (every layer holds one draw of layer 0's tokens).
+    Re-running the step rewrites the same bytes: the staged tokens come from ring slots that the
+    step does not write."""
+    import numpy as np
+    import torch
+
+    import paper_2607_20538_gb300 as cg
+    from paper_2607_20538_gb300 import synth
+    P = _Problem()
+    Tc = w.T_cap
+    params = cg.Params(**w.params)
+    full = cg.Shape(L=w.L, B=w.B, H=w.H, T=Tc, d=w.d, t0=0, T_cap=Tc)
+    app = cg.Shape(L=w.L, B=w.B, H=w.H, T=1, d=w.d, t0=Tc - 1, T_cap=Tc)
+    lay = cg.Shape(L=1, B=w.B, H=w.H, T=Tc - 1, d=w.d, t0=0, T_cap=Tc)
+    nc, ns, nr, nw = cg.kivi_stream_bytes(full, params)
+    nc1, ns1, nr1, _ = cg.kivi_stream_bytes(lay, params)
+    P.G = synth.gauges(w)
+    dG = torch.from_numpy(P.G.reshape(-1)).to(dev)
+    codes, scales, ring, work = cg.kivi_stream_alloc(full, params, device=dev)
+    threads = max(4, (os.cpu_count() or 8) // max(ws, 1))
+    dh = torch.from_numpy(synth.rolling_history_layer(w, threads=threads).reshape(-1).view(np.int16)).to(dev)
+    per_g = dG.numel() // w.L
+    for l in range(w.L):
+        cg.kivi_append(lay, params, dh, dG[l * per_g:(l + 1) * per_g], codes[l * nc1:(l + 1) * nc1],
+                       scales[l * ns1 // 4:(l + 1) * ns1 // 4], ring[l * nr1 // 2:(l + 1) * nr1 // 2], None,
+                       stream=stream)
+    del dh
+    xnew = synth.rolling_new_token(w, threads=threads)
+    dnew = torch.from_numpy(xnew.reshape(-1).view(np.int16)).to(dev)
+    n_out = w.L * 2 * w.B * w.H * Tc * w.d
+    out = torch.empty(n_out, dtype=torch.int16, device=dev)
+    Gt, units = w.block, w.L * 2 * w.B * w.H
+    P.enc_bytes, P.dec_bytes = xnew.nbytes, 2 * n_out
+    grp_codes = units * Gt * w.d * w.bits // 8
+    grp_scales = w.L * w.B * w.H * (w.d + Gt * (w.d // Gt)) * 4
+    # staging: the group's tokens read from the ring and written to the workspace, read again
+    # by the quantizers; the new token in and into the ring
+    P.enc_alg = 2 * xnew.nbytes + 3 * units * Gt * w.d * 2 + grp_codes + grp_scales + P.G.nbytes
+    nq = (Tc - w.residual) // Gt * Gt
+    P.dec_alg = nc + ns + units * (Tc - nq) * w.d * 2 + P.G.nbytes + 2 * n_out
+    P.launches = 4 + 3
+    P.config = {"T_cap": Tc, "step": "KIVI stream: append 1 token per sequence at T_cap - 1 (completes a key "
+                                     "group), decode all T_cap tokens"}
+
+    def encode():
+        cg.kivi_append(app, params, dnew, dG, codes, scales, ring, work, stream=stream)
+
+    def decode():
+        cg.kivi_stream_decode(full, params, codes, scales, ring, dG, out, stream=stream)
+
+    P.encode, P.decode = encode, decode
+    hnew = torch.from_numpy(xnew.reshape(-1).view(np.int16)).pin_memory()
+    last = out.view(units, Tc, w.d)[:, Tc - 1, :]
+    hlast = torch.empty(last.shape, dtype=torch.int16).pin_memory()
+
+    def e2e_step():
+        dnew.copy_(hnew, non_blocking=True)
+        encode()
+        decode()
+        hlast.copy_(last, non_blocking=True)
+
+    P.e2e_step, P.h2d, P.d2h = e2e_step, hnew.numel() * 2, hlast.numel() * 2
+    P.e2e_bytes = P.enc_bytes + P.dec_bytes
+    return P
+
+
+def _setup(w, dev, ws, stream):
+    if w.T_cap:
+        return (_setup_kivi_stream if w.backend == 1 else _setup_rolling)(w, dev, ws, stream)
+    return _setup_cache(w, dev, ws, stream)
+
+
 def _time_problem(P, stream, steps: int, warmup: int, dev, ws: int, clock_dev: int):
     """Warm-up, then `steps` timed steps of problem P on `stream` (CUDA events per kernel and
     around the whole region, nvidia-smi clocks sampled during it)."""
@@ -438,7 +514,7 @@ PAPER_CONTEXT = {
 }
 
 # The other target workloads, timed in the same process after the headline one.
-EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "llama3_8b_tile")
+EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "kivi3_stream", "llama3_8b_tile")
 
 
 def run_cuda(args):
@@ -459,7 +535,7 @@ def run_cuda(args):
     clock_dev = dev if ws == 1 else local
     w = _workload(args)
     stream = torch.cuda.current_stream()
-    P = (_setup_rolling if w.T_cap else _setup_cache)(w, dev, ws, stream)
+    P = _setup(w, dev, ws, stream)
     t = _time_problem(P, stream, args.steps, args.warmup, dev, ws, clock_dev)
     ms_step = t["ms_step"]
     value = job_throughput(P.enc_bytes + P.dec_bytes, ws, ms_step)
@@ -524,7 +600,7 @@ def run_cuda(args):
     if not args.layers and not args.shape and not args.no_extra and args.workload == "llama3_8b":
         for name in EXTRA_WORKLOADS:
             we = synth.WORKLOADS[name]
-            Pe = (_setup_rolling if we.T_cap else _setup_cache)(we, dev, ws, stream)
+            Pe = _setup(we, dev, ws, stream)
             te = _time_problem(Pe, stream, args.extra_steps, 3, dev, ws, clock_dev)
             fig = _kernel_figures(Pe, te, peak)
             fig["steps"] = args.extra_steps

@@ -70,8 +70,9 @@ class Workload:
 
 
 # The cache workloads: a tiny case, a Llama-3-8B-shaped cache (per-token blocks, and the
-# paper's 16-token tiles), a Qwen/Mistral-shaped KIVI case, a Gemma-2-27B-shaped 6-bit case
-# and a rolling decode step over a 16k history.
+# paper's 16-token tiles), a Qwen/Mistral-shaped KIVI case (whole cache, and a KIVI decode loop
+# over a 32k history), a Gemma-2-27B-shaped 6-bit case and a rolling decode step over a 16k
+# history.
 WORKLOADS = {
     "tiny": Workload("tiny", L=1, B=1, H=2, T=256, d=64, group=16, backend=0, bits=4, block=32,
                      n_outlier=2, outlier_mult=10.0, sigma_v=0.3, kv_seed=1000, gauge_seed=2000),
@@ -84,6 +85,10 @@ WORKLOADS = {
     "gemma27b": Workload("gemma27b", L=46, B=2, H=16, T=8192, d=128, group=32, backend=0, bits=6,
                          block=32, n_outlier=8, outlier_mult=20.0, sigma_v=0.5, kv_seed=1003,
                          gauge_seed=2003),
+    # a KIVI decode loop over the Qwen-shaped cache: a 32k history, one token appended per step
+    "kivi3_stream": Workload("kivi3_stream", L=28, B=4, H=4, T=32768, d=128, group=64, backend=1, bits=3,
+                             block=128, residual=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,
+                             kv_seed=1002, gauge_seed=2002, T_cap=32768),
     # the paper's block-uniform block shape on the 8B cache: one range per 16-token x d tile
     "llama3_8b_tile": Workload("llama3_8b_tile", L=32, B=1, H=8, T=8192, d=128, group=128, backend=3,
                                bits=4, block=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,

@@ -145,3 +145,52 @@ def test_rolling_full_size_step():
         su = _sub_bu(scales.view(torch.int32), wu, Tc, l, b, h, w.d // w.block).view(np.uint16)
         ou = out.view(w.L, 2, w.B, w.H, Tc, w.d)[l, :, b, h].contiguous().cpu().numpy().view(np.uint16).ravel()
         _check_unit(wu, G, np.ascontiguousarray(xu), l, h, cu, su, np.zeros(0, np.uint16), ou)
+
+
+def test_kivi_stream_full_size_step():
+    """KIVI decode-loop step at full size (the benchmark's kivi3_stream): a 32k-token stream per
+    sequence (28 layers, batch 4, 4 heads), one appended token that completes a key group, then
+    the whole history decoded; sampled units against the batch oracle of all 32768 tokens."""
+    from cgcheck import stream_to_batch
+    w = synth.WORKLOADS["kivi3_stream"]
+    Tc = w.T_cap
+    G = synth.gauges(w)
+    dG = torch.from_numpy(G.reshape(-1)).cuda()
+    params = cg.Params(**w.params)
+    hist1 = synth.rolling_history_layer(w, threads=16)          # [1][2][B][H][Tc-1][d]
+    xnew = synth.rolling_new_token(w, threads=16)               # [L][2][B][H][1][d]
+    full = cg.Shape(L=w.L, B=w.B, H=w.H, T=Tc, d=w.d, t0=0, T_cap=Tc)
+    codes, scales, ring, work = cg.kivi_stream_alloc(full, params)
+    lay = cg.Shape(L=1, B=w.B, H=w.H, T=Tc - 1, d=w.d, t0=0, T_cap=Tc)
+    nc1, ns1, nr1, _ = cg.kivi_stream_bytes(lay, params)
+    dh = torch.from_numpy(hist1.reshape(-1).view(np.int16)).cuda()
+    per_g = dG.numel() // w.L
+    for l in range(w.L):
+        cg.kivi_append(lay, params, dh, dG[l * per_g:(l + 1) * per_g], codes[l * nc1:(l + 1) * nc1],
+                       scales[l * ns1 // 4:(l + 1) * ns1 // 4], ring[l * nr1 // 2:(l + 1) * nr1 // 2])
+    del dh
+    app = cg.Shape(L=w.L, B=w.B, H=w.H, T=1, d=w.d, t0=Tc - 1, T_cap=Tc)
+    cg.kivi_append(app, params, torch.from_numpy(xnew.reshape(-1).view(np.int16)).cuda(), dG, codes, scales, ring,
+                   work)
+    out = torch.empty(w.L * 2 * w.B * w.H * Tc * w.d, dtype=torch.int16, device="cuda")
+    cg.kivi_stream_decode(full, params, codes, scales, ring, dG, out)
+    assert cg.get_status() == 0
+    # one unit's slices of the stream buffers, as a 1-layer, 1-sequence, 1-head stream
+    w1 = w.replace(L=1, B=1, H=1, T=Tc, T_cap=Tc)
+    Gt, pay = w.block, w.block * w.bits // 8
+    ncap = oracle.kivi_nq(Tc, w.residual, Gt)
+    kc, vc = (ncap // Gt) * w.d * pay, ncap * (w.d // Gt) * pay     # code bytes per (b, h)
+    ks, vs = (ncap // Gt) * w.d, ncap * (w.d // Gt)                 # scale pairs (u32) per (b, h)
+    c8, s32 = codes.view(torch.uint8), scales.view(torch.int32)
+    BH = w.B * w.H
+    W = w.residual + w.block
+    for (l, b, h) in _units(w):
+        bh = b * w.H + h
+        lc, ls = c8[l * nc1:(l + 1) * nc1], s32[l * ns1 // 4:(l + 1) * ns1 // 4]
+        cu = torch.cat([lc[bh * kc:(bh + 1) * kc], lc[BH * kc + bh * vc:BH * kc + (bh + 1) * vc]]).cpu().numpy()
+        su = torch.cat([ls[bh * ks:(bh + 1) * ks], ls[BH * ks + bh * vs:BH * ks + (bh + 1) * vs]]).cpu().numpy()
+        ru = ring.view(w.L, 2, w.B, w.H, W, w.d)[l, :, b, h].contiguous().cpu().numpy()
+        c1, s1, r1 = stream_to_batch(w1, Tc, Tc, cu, su.view(np.uint16), ru.view(np.uint16))
+        xu = np.concatenate([hist1[0:1, :, b:b + 1, h:h + 1], xnew[l:l + 1, :, b:b + 1, h:h + 1]], axis=4)
+        ou = out.view(w.L, 2, w.B, w.H, Tc, w.d)[l, :, b, h].contiguous().cpu().numpy().view(np.uint16).ravel()
+        _check_unit(w1.replace(T_cap=0), G, np.ascontiguousarray(xu), l, h, c1, s1, r1, ou)
