@@ -6,7 +6,7 @@ imports it. The arithmetic lives in ``cg_oracle.c`` (plain C, compiled with
 ``-ffp-contract=off`` and no fast-math); this module only marshals numpy arrays.
 
 Pins: ``tests/test_oracle_pins.py``, ``tests/test_oracle_tile_pins.py`` and
-``tests/test_oracle_stream_pins.py`` (closed forms,
+``tests/test_oracle_stream_pins.py``, ``tests/test_oracle_attention_pins.py`` (closed forms,
 brute force, worked examples, library routines). No function here is "parity unpinned".
 """
 from __future__ import annotations
@@ -77,6 +77,8 @@ def lib():
         L.cgo_kivi_append.argtypes = [P(_Shape), P(_Params), vp, vp, vp, vp, vp, ctypes.c_int, P(ctypes.c_int32)]
         L.cgo_kivi_stream_decode.restype = ctypes.c_int
         L.cgo_kivi_stream_decode.argtypes = [P(_Shape), P(_Params), vp, vp, vp, vp, vp, ctypes.c_int]
+        L.cgo_attention.restype = ctypes.c_int
+        L.cgo_attention.argtypes = [ctypes.c_int] * 6 + [vp, vp, ctypes.c_double, vp]
         L.cgo_gauge_coord.restype = ctypes.c_float
         L.cgo_gauge_coord.argtypes = [vp, vp, ctypes.c_int]
         _lib = L
@@ -223,3 +225,19 @@ def kivi_stream_decode(shape: dict, params: dict, codes, scales, ring, gauges, *
     if rc:
         raise ValueError(f"oracle kivi_stream_decode rc={rc}")
     return out
+
+
+# ---------------------------------------------------------------- attention
+def attention(shape: dict, n_rep: int, q_bf16: np.ndarray, xhat: np.ndarray, scale: float) -> np.ndarray:
+    """fp64 softmax attention of one query per sequence (n_rep query heads per KV head) over the
+    decoded cache xhat [L][2][B][H][T][d]; q bf16 [L][B][H][n_rep][d]. Returns [L][B][H][n_rep][d]."""
+    L, B, H, T, d = (shape[k] for k in ("L", "B", "H", "T", "d"))
+    q = np.ascontiguousarray(q_bf16).view(np.uint16)
+    assert q.size == L * B * H * n_rep * d
+    xh = np.ascontiguousarray(xhat, np.float64)
+    assert xh.size == L * 2 * B * H * T * d
+    out = np.zeros(L * B * H * n_rep * d, np.float64)
+    rc = lib().cgo_attention(L, B, H, T, d, n_rep, _ptr(q), _ptr(xh), float(scale), _ptr(out))
+    if rc:
+        raise ValueError(f"oracle attention rc={rc}")
+    return out.reshape(L, B, H, n_rep, d)

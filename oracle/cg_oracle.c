@@ -19,7 +19,7 @@
  * the single IEEE operation it reads as.
  *
  * Status of the pins (tests/test_oracle_pins.py, tests/test_oracle_tile_pins.py,
- * tests/test_oracle_stream_pins.py): every
+ * tests/test_oracle_stream_pins.py, tests/test_oracle_attention_pins.py): every
  * exported function is pinned against closed forms, brute force, worked examples or
  * library routines; none is "parity unpinned".
  */
@@ -855,5 +855,50 @@ int cgo_kivi_stream_decode(const cgo_shape* s, const cgo_params* p, const uint8_
     P.n_units = (int64_t)s->L * s->B * s->H;
     P.fn = kivi_stream_decode_unit;
     run_pool(&P, nthreads);
+    return CGO_OK;
+}
+
+/* ------------------------------------------------------------------------------ */
+/* Attention over the recovered cache (Fig. 1: the inverse gauge restores the cache  */
+/* before attention; standard softmax attention, grouped queries, Sec. 3)          */
+/* ------------------------------------------------------------------------------ */
+/* One decoding query per sequence: n_rep query heads share each KV head (grouped-query
+ * attention; n_rep = 1 is multi-head attention). For query head r of KV head h:
+ *   s_t = scale * sum_c q[c] Khat[t][c],  p_t = exp(s_t - max_t s_t) / sum_t exp(...),
+ *   o[c] = sum_t p_t Vhat[t][c],
+ * all in fp64, with Khat, Vhat the decoded cache xhat [L][2][B][H][T][d] (s = 0 keys, 1 values)
+ * and q bf16 [L][B][H][n_rep][d]. out: fp64 [L][B][H][n_rep][d]. */
+int cgo_attention(int L, int B, int H, int T, int d, int n_rep, const uint16_t* q, const double* xhat,
+                  double scale, double* out)
+{
+    if (L < 1 || B < 1 || H < 1 || T < 1 || d < 1 || n_rep < 1) return CGO_EINVAL;
+    double* s = (double*)malloc(sizeof(double) * (size_t)T);
+    for (int l = 0; l < L; l++)
+        for (int b = 0; b < B; b++)
+            for (int h = 0; h < H; h++) {
+                const double* K = xhat + ((((size_t)l * 2 + 0) * B + b) * H + h) * (size_t)T * d;
+                const double* V = xhat + ((((size_t)l * 2 + 1) * B + b) * H + h) * (size_t)T * d;
+                for (int r = 0; r < n_rep; r++) {
+                    size_t qi = ((((size_t)l * B + b) * H + h) * n_rep + r) * (size_t)d;
+                    double mx = -INFINITY;
+                    for (int t = 0; t < T; t++) {
+                        double acc = 0.0;
+                        for (int c = 0; c < d; c++) acc += (double)cgo_bf16_to_f32(q[qi + c]) * K[(size_t)t * d + c];
+                        s[t] = scale * acc;
+                        if (s[t] > mx) mx = s[t];
+                    }
+                    double z = 0.0;
+                    for (int t = 0; t < T; t++) {
+                        s[t] = exp(s[t] - mx);
+                        z += s[t];
+                    }
+                    for (int c = 0; c < d; c++) {
+                        double acc = 0.0;
+                        for (int t = 0; t < T; t++) acc += s[t] * V[(size_t)t * d + c];
+                        out[qi + c] = acc / z;
+                    }
+                }
+            }
+    free(s);
     return CGO_OK;
 }
