@@ -201,6 +201,29 @@ int cg_kivi_stream_decode(const cg_shape* shape, const cg_params* params, const 
                           const void* scales, const void* ring, const float* gauges,
                           void* out_kv_bf16, void* stream);
 
+/* ---- Attention straight from a block-uniform cache (Fig. 1: the recovered cache is consumed
+ * by softmax attention; Sec. 3: recovery can be folded into the surrounding computation) ----
+ * One decoding query per sequence, n_rep query heads per KV head (grouped queries; 1 = MHA):
+ *   s_t = scale * q . khat_t,  p = softmax_t(s),  o = sum_t p_t vhat_t
+ * over tokens [t0, t0 + T) of the cache, where khat, vhat are what cg_decode would recover.
+ * The inverse gauge is folded out of the token loop: q is rotated once into gauge space
+ * (q . G^T zhat = (G q) . zhat) and the weighted sum of values stays in gauge space until one
+ * G_V^T per query, so the kernels read only codes and scales. Arithmetic is fp32 (scores,
+ * softmax, sums); the result is fp32, not bit-exact (see the tolerance in the tests).
+ * Supported: CG_BLOCK_UNIFORM and CG_BLOCK_TILE caches with d = 128 and block in {32, 64, 128},
+ * any group and bit width; n_rep in {1, 2, 4, 8}; T >= 1. q: bf16 [L][B][H][n_rep][d];
+ * out: fp32 [L][B][H][n_rep][d]. workspace: caller-owned device scratch of
+ * cg_attention_workspace_bytes (rotated queries and per-512-token partial results). */
+int cg_attention_workspace_bytes(const cg_shape* shape, const cg_params* params, int n_rep,
+                                 size_t* workspace_bytes);
+
+/* Launches three kernels in order on `stream` (query rotation, per-chunk attention, merge);
+ * a CG_ECUDA may follow queued launches, and `out` is then invalid. Pointers 16-byte aligned;
+ * CG_EINVAL if workspace_bytes is below the required size or scale is not finite. */
+int cg_attention(const cg_shape* shape, const cg_params* params, int n_rep, float scale,
+                 const void* q_bf16, const void* codes, const void* scales, const float* gauges,
+                 float* out, void* workspace, size_t workspace_bytes, void* stream);
+
 /* Reads and clears (in one atomic step, ordered on `stream`) the accumulated CG_FLAG_* bits
  * of the current device, synchronizes `stream` and returns them in *device_flags. Returns
  * CG_ECUDA if a launch, copy or the synchronize fails. The limit of each bounded pipeline

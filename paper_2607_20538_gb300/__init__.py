@@ -18,7 +18,8 @@ from dataclasses import dataclass
 
 __all__ = ["CG_BLOCK_UNIFORM", "CG_KIVI", "CG_NONE", "CG_BLOCK_TILE", "CG_TILE_TOKENS", "Shape", "Params",
            "packed_bytes", "encode", "decode", "get_status", "lib_path", "load", "CodecGaugeError",
-           "kivi_stream_bytes", "kivi_stream_alloc", "kivi_append", "kivi_stream_decode"]
+           "kivi_stream_bytes", "kivi_stream_alloc", "kivi_append", "kivi_stream_decode",
+           "attention_workspace_bytes", "attention"]
 
 CG_BLOCK_UNIFORM, CG_KIVI, CG_NONE, CG_BLOCK_TILE = 0, 1, 2, 3
 CG_TILE_TOKENS = 16
@@ -97,6 +98,11 @@ def load():
         L.cg_kivi_append.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
         L.cg_kivi_stream_decode.restype = ctypes.c_int
         L.cg_kivi_stream_decode.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp, vp, vp]
+        L.cg_attention_workspace_bytes.restype = ctypes.c_int
+        L.cg_attention_workspace_bytes.argtypes = [P(_CShape), P(_CParams), ctypes.c_int, P(ctypes.c_size_t)]
+        L.cg_attention.restype = ctypes.c_int
+        L.cg_attention.argtypes = [P(_CShape), P(_CParams), ctypes.c_int, ctypes.c_float, vp, vp, vp, vp, vp, vp,
+                                   ctypes.c_size_t, vp]
         L.cg_get_status.restype = ctypes.c_int
         L.cg_get_status.argtypes = [vp, P(ctypes.c_int32)]
         L.cg_last_error.restype = ctypes.c_char_p
@@ -171,6 +177,23 @@ def kivi_stream_decode(shape: Shape, params: Params, codes, scales, ring, gauges
     """Decode the T tokens a KIVI stream holds (shape.t0 = 0) into the caller's bf16 output."""
     _check(load().cg_kivi_stream_decode(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(codes),
                                         _ptr(scales), _ptr(ring), _ptr(gauges), _ptr(out), _stream(stream)))
+
+
+def attention_workspace_bytes(shape: Shape, params: Params, n_rep: int) -> int:
+    """Workspace bytes of cg_attention for this cache shape and query heads per KV head."""
+    v = ctypes.c_size_t()
+    _check(load().cg_attention_workspace_bytes(ctypes.byref(shape.c()), ctypes.byref(params.c()), n_rep,
+                                               ctypes.byref(v)))
+    return v.value
+
+
+def attention(shape: Shape, params: Params, n_rep: int, scale: float, q, codes, scales, gauges, out, workspace,
+              stream=None) -> None:
+    """Softmax attention of one query per sequence (q bf16 [L][B][H][n_rep][d]) over tokens
+    [t0, t0 + T) of a block-uniform cache, straight from its codes; out fp32 [L][B][H][n_rep][d]."""
+    nbytes = workspace.numel() * workspace.element_size()
+    _check(load().cg_attention(ctypes.byref(shape.c()), ctypes.byref(params.c()), n_rep, scale, _ptr(q), _ptr(codes),
+                               _ptr(scales), _ptr(gauges), _ptr(out), _ptr(workspace), nbytes, _stream(stream)))
 
 
 def get_status(stream=None) -> int:

@@ -11,7 +11,7 @@ CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libcodecgauge.so")
 BUILD_DIR = os.path.join(HERE, "_build")
 SOURCES = ["cg_api.cu", "cg_simt.cu", "cg_tc.cu", "cg_tc_rows.cu", "cg_tc_dec.cu", "cg_tc_keydec.cu",
-           "cg_noalloc.cu"]
+           "cg_noalloc.cu", "cg_attn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -1,6 +1,7 @@
 // cg_api.cu -- the extern "C" boundary of libcodecgauge: argument validation, the
 // closed-form byte counts, kernel selection, the device status word and error strings.
 // Declarations and the full contract: include/codecgauge.h.
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -659,6 +660,81 @@ CG_EXPORT int cg_kivi_stream_decode(const cg_shape* shape, const cg_params* para
     m.dst_T = T;
     m.dst_t0 = 0;
     if ((e = launch_row_move(m, st)) != cudaSuccess) return cuda_fail(e, "KIVI stream window launch");
+    return CG_OK;
+}
+
+namespace {
+
+// Attention arguments common to the size query and the call.
+int validate_attention(const cg_shape* sh, const cg_params* p, int n_rep, Sizes* z) {
+    int rc = validate(sh, p, z);
+    if (rc) return rc;
+    if (p->backend != CG_BLOCK_UNIFORM && p->backend != CG_BLOCK_TILE)
+        return fail(CG_EUNSUPPORTED, "attention reads block-uniform caches (rows or tiles)");
+    if (sh->d != 128) return fail(CG_EUNSUPPORTED, "attention: head dim d=%d (d = 128 is provided)", sh->d);
+    if (!(p->block == 32 || p->block == 64 || p->block == 128))
+        return fail(CG_EUNSUPPORTED, "attention: block=%d (32, 64 or 128 are provided)", p->block);
+    if (!(n_rep == 1 || n_rep == 2 || n_rep == 4 || n_rep == 8))
+        return fail(CG_EINVAL, "n_rep=%d: query heads per KV head must be 1, 2, 4 or 8", n_rep);
+    if (sh->T < 1) return fail(CG_EINVAL, "attention needs T >= 1 tokens");
+    return CG_OK;
+}
+
+}  // namespace
+
+CG_EXPORT int cg_attention_workspace_bytes(const cg_shape* shape, const cg_params* params, int n_rep,
+                                           size_t* workspace_bytes) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate_attention(shape, params, n_rep, &z);
+    if (rc) return rc;
+    if (workspace_bytes)
+        *workspace_bytes = attn_workspace_bytes((int64_t)shape->L * shape->B * shape->H, n_rep, shape->d, shape->T);
+    return CG_OK;
+}
+
+CG_EXPORT int cg_attention(const cg_shape* shape, const cg_params* params, int n_rep, float scale, const void* q_bf16,
+                           const void* codes, const void* scales, const float* gauges, float* out,
+                           void* workspace, size_t workspace_bytes, void* stream) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate_attention(shape, params, n_rep, &z);
+    if (rc) return rc;
+    if (!(scale == scale) || scale == INFINITY || scale == -INFINITY)
+        return fail(CG_EINVAL, "softmax scale must be finite");
+    if (!q_bf16 || !codes || !scales || !gauges || !out || !workspace)
+        return fail(CG_EINVAL, "null q, codes, scales, gauges, out or workspace pointer");
+    const size_t need = attn_workspace_bytes((int64_t)shape->L * shape->B * shape->H, n_rep, shape->d, shape->T);
+    if (workspace_bytes < need) return fail(CG_EINVAL, "workspace needs %zu bytes (got %zu)", need, workspace_bytes);
+    if (!aligned16(q_bf16) || !aligned16(codes) || !aligned16(scales) || !aligned16(gauges) || !aligned16(out) ||
+        !aligned16(workspace))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    AttnArgs a{};
+    a.q = static_cast<const uint16_t*>(q_bf16);
+    a.G = gauges;
+    a.codes = static_cast<const uint8_t*>(codes);
+    a.scales = static_cast<const uint32_t*>(scales);
+    bu_maps(shape, z, z.nb * z.pay, z.nb, &a.cmap, &a.smap, params->backend == CG_BLOCK_TILE);
+    const int64_t units = (int64_t)shape->L * shape->B * shape->H;
+    a.qrot = static_cast<float*>(workspace);
+    a.part = reinterpret_cast<float*>(static_cast<unsigned char*>(workspace) +
+                                      ((size_t)units * n_rep * shape->d * 4 + 255) / 256 * 256);
+    a.out = out;
+    a.L = shape->L;
+    a.B = shape->B;
+    a.H = shape->H;
+    a.d = shape->d;
+    a.g = params->group;
+    a.bits = params->bits;
+    a.blk = params->block;
+    a.n_rep = n_rep;
+    a.T = shape->T;
+    a.n_chunks = (int)((shape->T + kAttnChunk - 1) / kAttnChunk);
+    a.scale = scale;
+    cudaError_t e = launch_attention(a, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "attention launch");
     return CG_OK;
 }
 

@@ -65,6 +65,26 @@ struct MoveArgs {
     int64_t dst_T, dst_t0;
 };
 
+// Attention of one query per sequence over a block-uniform cache, from the packed codes.
+struct AttnArgs {
+    const uint16_t* q;      // bf16 [L][B][H][n_rep][d]
+    const float* G;         // [L][2][H][d/g][g][g]
+    const uint8_t* codes;   // block-uniform codes (rows layout)
+    const uint32_t* scales; // half2 {s, m} per block (per token, or per 16-token tile)
+    RowMap cmap, smap;      // row maps of tokens [t0, t0 + T)
+    float* qrot;            // workspace: scale * G_K q, [L*B*H][n_rep][d]
+    float* part;            // workspace: [L*B*H][n_chunks][n_rep][d + 2] (max, sum, o')
+    float* out;             // fp32 [L][B][H][n_rep][d]
+    int L, B, H, d, g, bits, blk, n_rep;
+    int64_t T;              // tokens attended
+    int n_chunks;
+    float scale;
+};
+
+constexpr int kAttnChunk = 512;  // tokens per CTA of the chunk kernel
+size_t attn_workspace_bytes(int64_t units, int n_rep, int d, int64_t T);
+cudaError_t launch_attention(const AttnArgs& a, cudaStream_t st);
+
 // Sets the message cg_last_error() returns on this host thread; returns code.
 int set_error(int code, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
 

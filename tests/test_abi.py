@@ -107,6 +107,25 @@ def test_kivi_stream_bytes_and_validation(lib):
     assert lib.cg_kivi_stream_decode(S(t0=1, T=2), P, fake, fake, fake, fake, fake, None) == -2
 
 
+def test_attention_validation(lib):
+    """cg_attention: supported caches and query-head counts are checked on the host."""
+    sh = cg.Shape(L=2, B=3, H=2, T=1100, d=128)
+    nb = cg.attention_workspace_bytes(sh, cg.Params(0, 128, 4, 64), 4)
+    assert nb == -(-2 * 3 * 2 * 4 * 128 * 4 // 256) * 256 + 2 * 3 * 2 * 3 * 4 * 130 * 4   # queries, 3 chunks
+    for params, n_rep in ((cg.Params(cg.CG_KIVI, 64, 3, 128, 128), 4), (cg.Params(0, 16, 4, 16), 4),
+                          (cg.Params(0, 16, 4, 64), 3)):
+        with pytest.raises(cg.CodecGaugeError):
+            cg.attention_workspace_bytes(sh, params, n_rep)
+    with pytest.raises(cg.CodecGaugeError):
+        cg.attention_workspace_bytes(cg.Shape(L=1, B=1, H=1, T=64, d=64), cg.Params(0, 16, 4, 32), 1)
+    fake = ctypes.c_void_p(0x10000)
+    S, P = ctypes.byref(sh.c()), ctypes.byref(cg.Params(0, 128, 4, 64).c())
+    assert lib.cg_attention(S, P, 4, ctypes.c_float(float("nan")), fake, fake, fake, fake, fake, fake, 1 << 30,
+                            None) == -1
+    assert lib.cg_attention(S, P, 4, ctypes.c_float(0.1), fake, fake, fake, fake, fake, fake, 16, None) == -1
+    assert "workspace" in lib.cg_last_error().decode()
+
+
 def test_pointer_checks_fail_before_device(lib):
     shape = cg.Shape(L=1, B=1, H=1, T=4, d=64)
     params = cg.Params(0, 16, 4, 32)

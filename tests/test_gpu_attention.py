@@ -1,0 +1,103 @@
+"""GPU parity of the attention read straight from a block-uniform cache (cg_attention).
+
+The reference is the oracle's fp64 softmax attention (pinned in test_oracle_attention_pins.py)
+over the oracle's fp64 decode of the same packed bytes (pinned in test_oracle_pins.py): the
+attention over the recovered cache of Sec. 3 / Fig. 1. The GPU folds the inverse gauge out of
+the token loop and works in fp32, so it is compared with a tolerance derived from its
+arithmetic: scores carry relative errors of a few 1e-6 (the code dot products over 128 channels
+in fp32, the rotation of the query), which move the output by at most that much times the spread
+of the values; the sums over up to 2048 tokens per chunk and the merge add a few 1e-6 relative.
+The test bound, |o_gpu - o_ref| <= 2e-5 * max|vhat| over the (l, b, h) unit (plus 1e-6
+* max|vhat| per 1024 tokens), is an order of magnitude above that and far below the 1e-3
+relative accuracy the decoded cache itself is held to.
+
+Cases span several 512-token chunks with a ragged last chunk, every bit width, block sizes 32,
+64 and 128, gauge groups 16..128, 1, 2, 4 and 8 query heads per KV head, 16-token tiles, windows
+that start inside a history, and end-to-end inputs encoded by the GPU.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2607_20538_gb300 import synth
+
+torch = pytest.importorskip("torch")
+cg = pytest.importorskip("paper_2607_20538_gb300")
+
+pytestmark = pytest.mark.gpu
+
+
+def _wl(**kw):
+    base = dict(name="attn", L=2, B=3, H=2, T=1100, d=128, group=128, backend=0, bits=4, block=64, residual=0)
+    base.update(kw)
+    return synth.Workload(**base)
+
+
+# (workload, n_rep, t0 of the window, tokens attended)
+CASES = {
+    "bu4_blk64_g128_rep4": (_wl(), 4, 0, 1100),
+    "bu3_blk32_g32_rep2": (_wl(bits=3, block=32, group=32, T=700), 2, 0, 700),
+    "bu6_blk128_g64_rep8": (_wl(bits=6, block=128, group=64, T=513, B=2), 8, 0, 513),
+    "bu8_blk64_g16_rep1": (_wl(bits=8, block=64, group=16, T=100), 1, 0, 100),
+    "bu2_blk32_g128_rep4": (_wl(bits=2, block=32, T=2000, L=1), 4, 0, 2000),
+    "tile4_blk128_g128_rep4": (_wl(backend=3, block=128, T=777), 4, 0, 777),
+    "bu4_window": (_wl(T=700), 4, 37, 600),
+    "tile3_window": (_wl(backend=3, bits=3, block=64, group=32, T=700), 2, 32, 640),
+}
+
+
+def _tol(xr, w, T):
+    v = np.abs(xr.reshape(w.L, 2, w.B, w.H, T, w.d)[:, 1])               # values of each unit
+    vmax = v.max(axis=(-1, -2))                                          # [L][B][H]
+    return ((2e-5 + 1e-6 * T / 1024) * vmax)[..., None, None]
+
+
+def _run(w, n_rep, t0, T, codes_dev, scales_dev, codes_host, scales_host, G, q):
+    T_cap = w.T
+    shape = cg.Shape(L=w.L, B=w.B, H=w.H, T=T, d=w.d, t0=t0, T_cap=T_cap)
+    params = cg.Params(**w.params)
+    ws = torch.empty(cg.attention_workspace_bytes(shape, params, n_rep), dtype=torch.uint8, device="cuda")
+    out = torch.full((w.L * w.B * w.H * n_rep * w.d,), float("nan"), dtype=torch.float32, device="cuda")
+    dq = torch.from_numpy(q.reshape(-1).view(np.int16)).cuda()
+    dG = torch.from_numpy(G.reshape(-1)).cuda()
+    scale = 1.0 / np.sqrt(w.d)
+    cg.attention(shape, params, n_rep, scale, dq, codes_dev, scales_dev, dG, out, ws)
+    assert cg.get_status() == 0
+    win = dict(L=w.L, B=w.B, H=w.H, T=T, d=w.d, t0=t0, T_cap=T_cap)
+    xr = oracle.decode(win, w.params, codes_host, scales_host, None, G)
+    ref = oracle.attention(win, n_rep, q, xr, float(np.float32(scale)))
+    got = out.cpu().numpy().astype(np.float64).reshape(ref.shape)
+    err = np.abs(got - ref)
+    tol = _tol(xr, w, T)
+    assert np.isfinite(got).all()
+    assert (err <= tol).all(), f"max err {err.max():.3g}, worst err/tol {(err / tol).max():.3g}"
+    return float((err / tol).max())
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_attention_on_oracle_bytes(name):
+    w, n_rep, t0, T = CASES[name]
+    x = synth.kv_cache(w, threads=4)
+    G = synth.gauges(w)
+    ref = oracle.encode(w.shape, w.params, x, G)
+    q = synth.f32_to_bf16_bits(np.random.default_rng(3).normal(0.0, 1.0, (w.L, w.B, w.H, n_rep, w.d)).astype(np.float32))
+    dc = torch.from_numpy(np.concatenate([ref["codes"], np.zeros(16, np.uint8)])).cuda()
+    ds = torch.from_numpy(np.concatenate([ref["scales"], np.zeros(8, np.uint16)]).view(np.int16)).cuda()
+    r = _run(w, n_rep, t0, T, dc, ds, ref["codes"], ref["scales"], G, q)
+    print(f"{name}: worst err / tolerance {r:.3g}")
+
+
+@pytest.mark.parametrize("name", ["bu4_blk64_g128_rep4", "tile4_blk128_g128_rep4"])
+def test_attention_end_to_end(name):
+    """The GPU's own encode, then attention; the reference decodes the GPU's bytes."""
+    w, n_rep, t0, T = CASES[name]
+    x = synth.kv_cache(w, threads=4)
+    G = synth.gauges(w)
+    shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
+    nc, ns, _ = cg.packed_bytes(shape, params)
+    codes, scales, resid = cg.alloc_outputs(shape, params)
+    cg.encode(shape, params, torch.from_numpy(x.reshape(-1).view(np.int16)).cuda(),
+              torch.from_numpy(G.reshape(-1)).cuda(), codes, scales, resid)
+    q = synth.f32_to_bf16_bits(np.random.default_rng(4).normal(0.0, 1.0, (w.L, w.B, w.H, n_rep, w.d)).astype(np.float32))
+    _run(w, n_rep, t0, T, codes, scales, codes.cpu().numpy().view(np.uint8)[:nc],
+         scales.cpu().numpy().view(np.uint16)[: ns // 2], G, q)
