@@ -344,26 +344,49 @@ def _setup_rolling(w, dev, ws, stream):
     P.dec_alg = nc + ns + P.G.nbytes + 2 * n_out
     P.launches = 2
     P.config = {"T_cap": Tc, "step": "append 1 token per sequence at T_cap - 1, decode all T_cap tokens"}
+    n_rep = w.extra.get("n_rep", 0)
+    if n_rep:
+        # the step's second half is attention of one query per sequence over the whole history,
+        # read straight from the codes (no bf16 cache written)
+        del out
+        nq = w.L * w.B * w.H * n_rep * w.d
+        dq = torch.from_numpy(synth.f32_to_bf16_bits(
+            np.random.default_rng(w.kv_seed + 900).normal(0.0, 1.0, nq).astype(np.float32)).view(np.int16)).to(dev)
+        out = torch.empty(nq, dtype=torch.float32, device=dev)
+        work = torch.empty(cg.attention_workspace_bytes(full, params, n_rep), dtype=torch.uint8, device=dev)
+        P.dec_bytes = 2 * n_out  # bf16 bytes of the cache the attention reads through its codes
+        P.dec_alg = nc + ns + P.G.nbytes + dq.numel() * 2 + nq * 4
+        P.launches = 1 + 3
+        P.config = {"T_cap": Tc, "n_rep": n_rep,
+                    "step": "append 1 token per sequence at T_cap - 1, then attention of 1 query per sequence "
+                            f"({n_rep} query heads per KV head) over all T_cap tokens, from the codes"}
+        scale = 1.0 / float(np.sqrt(w.d))
+
+        def decode():
+            cg.attention(full, params, n_rep, scale, dq, codes, scales, dG, out, work, stream=stream)
+
+        last = out
+    else:
+        def decode():
+            cg.decode(full, params, codes, scales, None, dG, out, stream=stream)
+
+        last = out.view(w.L * 2 * w.B * w.H, Tc, w.d)[:, Tc - 1, :]
 
     def encode():
         cg.encode(app, params, dnew, dG, codes, scales, None, stream=stream)
 
-    def decode():
-        cg.decode(full, params, codes, scales, None, dG, out, stream=stream)
-
     P.encode, P.decode = encode, decode
     hnew = torch.from_numpy(xnew.reshape(-1).view(np.int16)).pin_memory()
-    last = out.view(w.L * 2 * w.B * w.H, Tc, w.d)[:, Tc - 1, :]
-    hlast = torch.empty(last.shape, dtype=torch.int16).pin_memory()
+    hlast = torch.empty(last.shape, dtype=last.dtype).pin_memory()
 
     def e2e_step():
-        # the new tokens in, the step, and the decoded newest token of every sequence out
+        # the new tokens in, the step, and the decoded newest token (or the attention output) out
         dnew.copy_(hnew, non_blocking=True)
         encode()
         decode()
         hlast.copy_(last, non_blocking=True)
 
-    P.e2e_step, P.h2d, P.d2h = e2e_step, hnew.numel() * 2, hlast.numel() * 2
+    P.e2e_step, P.h2d, P.d2h = e2e_step, hnew.numel() * 2, hlast.numel() * hlast.element_size()
     P.e2e_bytes = P.enc_bytes + P.dec_bytes
     return P
 
@@ -514,7 +537,7 @@ PAPER_CONTEXT = {
 }
 
 # The other target workloads, timed in the same process after the headline one.
-EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "kivi3_stream", "llama3_8b_tile")
+EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "rolling_attn", "kivi3_stream", "llama3_8b_tile")
 
 
 def run_cuda(args):

@@ -733,6 +733,8 @@ CG_EXPORT int cg_attention(const cg_shape* shape, const cg_params* params, int n
     a.T = shape->T;
     a.n_chunks = (int)((shape->T + kAttnChunk - 1) / kAttnChunk);
     a.scale = scale;
+    a.status = status;
+    a.wait_ns = pipe_wait_ns();
     cudaError_t e = launch_attention(a, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "attention launch");
     return CG_OK;

@@ -77,11 +77,15 @@ struct AttnArgs {
     float* out;             // fp32 [L][B][H][n_rep][d]
     int L, B, H, d, g, bits, blk, n_rep;
     int64_t T;              // tokens attended
-    int n_chunks;
+    int n_chunks;           // 256-token chunks of [t0, t0 + T)
+    int n_parts;            // partial results per (l, b, h), each over chunks_per_part chunks
+    int chunks_per_part;
     float scale;
+    int32_t* status;
+    uint64_t wait_ns;       // limit of the bounded waits on the chunk copies
 };
 
-constexpr int kAttnChunk = 512;  // tokens per CTA of the chunk kernel
+constexpr int kAttnChunk = 256;  // tokens per CTA of the chunk kernels
 size_t attn_workspace_bytes(int64_t units, int n_rep, int d, int64_t T);
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t st);
 

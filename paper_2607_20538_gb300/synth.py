@@ -85,6 +85,10 @@ WORKLOADS = {
     "gemma27b": Workload("gemma27b", L=46, B=2, H=16, T=8192, d=128, group=32, backend=0, bits=6,
                          block=32, n_outlier=8, outlier_mult=20.0, sigma_v=0.5, kv_seed=1003,
                          gauge_seed=2003),
+    # the rolling step with attention read straight from the codes (4 query heads per KV head)
+    "rolling_attn": Workload("rolling_attn", L=32, B=64, H=8, T=16384, d=128, group=128, backend=0, bits=4,
+                             block=64, n_outlier=4, outlier_mult=10.0, sigma_v=0.3, kv_seed=1004,
+                             gauge_seed=2004, T_cap=16384, extra={"n_rep": 4}),
     # a KIVI decode loop over the Qwen-shaped cache: a 32k history, one token appended per step
     "kivi3_stream": Workload("kivi3_stream", L=28, B=4, H=4, T=32768, d=128, group=64, backend=1, bits=3,
                              block=128, residual=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,

@@ -4,12 +4,15 @@ The reference is the oracle's fp64 softmax attention (pinned in test_oracle_atte
 over the oracle's fp64 decode of the same packed bytes (pinned in test_oracle_pins.py): the
 attention over the recovered cache of Sec. 3 / Fig. 1. The GPU folds the inverse gauge out of
 the token loop and works in fp32, so it is compared with a tolerance derived from its
-arithmetic: scores carry relative errors of a few 1e-6 (the code dot products over 128 channels
-in fp32, the rotation of the query), which move the output by at most that much times the spread
-of the values; the sums over up to 2048 tokens per chunk and the merge add a few 1e-6 relative.
-The test bound, |o_gpu - o_ref| <= 2e-5 * max|vhat| over the (l, b, h) unit (plus 1e-6
-* max|vhat| per 1024 tokens), is an order of magnitude above that and far below the 1e-3
-relative accuracy the decoded cache itself is held to.
+arithmetic. For 2- and 4-bit codes the contractions run on tensor cores with each code entering
+as the exact bf16 value 2^b + q: an MMA accumulates in fp32 with an error of a few u (u = 2^-24)
+of the accumulator per step, and the accumulated magnitude is up to 2^(b+1) sum_t w_t (the
+offset is removed afterwards), so over the 16 accumulation steps of a 512-token chunk the gauge
+-space value sum carries up to ~2e-4 of sum_t p_t s_t / sum_t p_t, i.e. of a quantization step
+(s <= range / 3 at b >= 2), that is a few 1e-5 of max|vhat|; the fp32 score dot products and the
+merge add a few 1e-6. The test bound, |o_gpu - o_ref| <= 1e-4 * max|vhat| over the (l, b, h)
+unit (plus 1e-5 * max|vhat| per 1024 tokens), sits above that and an order of magnitude below
+the 1e-3 relative accuracy the decoded cache itself is held to.
 
 Cases span several 512-token chunks with a ragged last chunk, every bit width, block sizes 32,
 64 and 128, gauge groups 16..128, 1, 2, 4 and 8 query heads per KV head, 16-token tiles, windows
@@ -49,7 +52,7 @@ CASES = {
 def _tol(xr, w, T):
     v = np.abs(xr.reshape(w.L, 2, w.B, w.H, T, w.d)[:, 1])               # values of each unit
     vmax = v.max(axis=(-1, -2))                                          # [L][B][H]
-    return ((2e-5 + 1e-6 * T / 1024) * vmax)[..., None, None]
+    return ((1e-4 + 1e-5 * T / 1024) * vmax)[..., None, None]
 
 
 def _run(w, n_rep, t0, T, codes_dev, scales_dev, codes_host, scales_host, G, q):
