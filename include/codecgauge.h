@@ -146,6 +146,22 @@ int cg_decode(const cg_shape* shape, const cg_params* params,
               const void* codes, const void* scales, const void* residual,
               const float* gauges, void* out_kv_bf16, void* stream);
 
+/* ---- Hadamard gauge by fast Walsh-Hadamard transform (the structured Hadamard control of
+ * Sec. 4.3) ----
+ * Encode / decode with the gauge G_{l,s,h,r} = H_g / sqrt(g) for every (l, s, h, r), H_g the
+ * Sylvester Hadamard matrix (H[i][j] = (-1)^popcount(i & j)), each entry stored as the fp32
+ * value +-c, c = fp32(1 / sqrt(g)) (1 / sqrt(g) computed in double, then rounded to fp32).
+ * No gauge tensor is read: the transform costs O(g log g) per group instead of g^2. The
+ * results are those of cg_encode / cg_decode given that gauge tensor: every product of the
+ * quantization rule is +-fl(c x_j), and its pairwise summation order over j is the butterfly
+ * order of the transform, so codes, scales and zeros are bit for bit the same; decode runs
+ * the transform in fp32. Block-uniform rows (CG_BLOCK_UNIFORM) only, any supported d, group,
+ * bits and block, with t0 / T_cap as for cg_encode; CG_EUNSUPPORTED for other backends. */
+int cg_encode_hadamard(const cg_shape* shape, const cg_params* params, const void* kv_bf16,
+                       void* out_codes, void* out_scales, void* stream);
+int cg_decode_hadamard(const cg_shape* shape, const cg_params* params, const void* codes,
+                       const void* scales, void* out_kv_bf16, void* stream);
+
 /* ---- KIVI streaming (Sec. 4.3 KIVI-style path; the growing cache of a decode loop) ----
  * A KIVI history of capacity T_cap tokens per (l, s, b, h) that grows by appends. Holding
  * T tokens, its first n_q(T) = max(0, floor((T - residual) / block)) * block tokens are

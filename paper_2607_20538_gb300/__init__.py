@@ -19,7 +19,7 @@ from dataclasses import dataclass
 __all__ = ["CG_BLOCK_UNIFORM", "CG_KIVI", "CG_NONE", "CG_BLOCK_TILE", "CG_TILE_TOKENS", "Shape", "Params",
            "packed_bytes", "encode", "decode", "get_status", "lib_path", "load", "CodecGaugeError",
            "kivi_stream_bytes", "kivi_stream_alloc", "kivi_append", "kivi_stream_decode",
-           "attention_workspace_bytes", "attention"]
+           "attention_workspace_bytes", "attention", "encode_hadamard", "decode_hadamard"]
 
 CG_BLOCK_UNIFORM, CG_KIVI, CG_NONE, CG_BLOCK_TILE = 0, 1, 2, 3
 CG_TILE_TOKENS = 16
@@ -103,6 +103,10 @@ def load():
         L.cg_attention.restype = ctypes.c_int
         L.cg_attention.argtypes = [P(_CShape), P(_CParams), ctypes.c_int, ctypes.c_float, vp, vp, vp, vp, vp, vp,
                                    ctypes.c_size_t, vp]
+        L.cg_encode_hadamard.restype = ctypes.c_int
+        L.cg_encode_hadamard.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp]
+        L.cg_decode_hadamard.restype = ctypes.c_int
+        L.cg_decode_hadamard.argtypes = [P(_CShape), P(_CParams), vp, vp, vp, vp]
         L.cg_get_status.restype = ctypes.c_int
         L.cg_get_status.argtypes = [vp, P(ctypes.c_int32)]
         L.cg_last_error.restype = ctypes.c_char_p
@@ -194,6 +198,18 @@ def attention(shape: Shape, params: Params, n_rep: int, scale: float, q, codes, 
     nbytes = workspace.numel() * workspace.element_size()
     _check(load().cg_attention(ctypes.byref(shape.c()), ctypes.byref(params.c()), n_rep, scale, _ptr(q), _ptr(codes),
                                _ptr(scales), _ptr(gauges), _ptr(out), _ptr(workspace), nbytes, _stream(stream)))
+
+
+def encode_hadamard(shape: Shape, params: Params, kv, codes, scales, stream=None) -> None:
+    """cg_encode with the Hadamard gauge H_g / sqrt(g), by fast Walsh-Hadamard transform."""
+    _check(load().cg_encode_hadamard(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(kv), _ptr(codes),
+                                     _ptr(scales), _stream(stream)))
+
+
+def decode_hadamard(shape: Shape, params: Params, codes, scales, out, stream=None) -> None:
+    """cg_decode with the Hadamard gauge H_g / sqrt(g), by fast Walsh-Hadamard transform."""
+    _check(load().cg_decode_hadamard(ctypes.byref(shape.c()), ctypes.byref(params.c()), _ptr(codes), _ptr(scales),
+                                     _ptr(out), _stream(stream)))
 
 
 def get_status(stream=None) -> int:

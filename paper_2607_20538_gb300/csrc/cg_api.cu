@@ -545,6 +545,54 @@ CG_EXPORT int cg_decode(const cg_shape* shape, const cg_params* params, const vo
     return CG_OK;
 }
 
+CG_EXPORT int cg_encode_hadamard(const cg_shape* shape, const cg_params* params, const void* kv_bf16,
+                                 void* out_codes, void* out_scales, void* stream) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate(shape, params, &z);
+    if (rc) return rc;
+    if (params->backend != CG_BLOCK_UNIFORM)
+        return fail(CG_EUNSUPPORTED, "the Hadamard transform path encodes block-uniform rows");
+    if (shape->T == 0) return CG_OK;
+    if (!kv_bf16 || !out_codes || !out_scales) return fail(CG_EINVAL, "null kv, codes or scales pointer");
+    if (!aligned16(kv_bf16) || !aligned16(out_codes) || !aligned16(out_scales))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    RowArgs a = row_args(shape, params, status);
+    a.x = static_cast<const uint16_t*>(kv_bf16);
+    a.codes = static_cast<uint8_t*>(out_codes);
+    a.scales = static_cast<uint32_t*>(out_scales);
+    bu_maps(shape, z, z.nb * z.pay, z.nb, &a.cmap, &a.smap);
+    cudaError_t e = launch_hadamard(a, true, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "Hadamard encode launch");
+    return CG_OK;
+}
+
+CG_EXPORT int cg_decode_hadamard(const cg_shape* shape, const cg_params* params, const void* codes,
+                                 const void* scales, void* out_kv_bf16, void* stream) {
+    t_err.clear();
+    Sizes z;
+    int rc = validate(shape, params, &z);
+    if (rc) return rc;
+    if (params->backend != CG_BLOCK_UNIFORM)
+        return fail(CG_EUNSUPPORTED, "the Hadamard transform path decodes block-uniform rows");
+    if (shape->T == 0) return CG_OK;
+    if (!codes || !scales || !out_kv_bf16) return fail(CG_EINVAL, "null codes, scales or output pointer");
+    if (!aligned16(codes) || !aligned16(scales) || !aligned16(out_kv_bf16))
+        return fail(CG_EINVAL, "pointers must be 16-byte aligned");
+    int32_t* status = nullptr;
+    if ((rc = status_ptr(&status))) return rc;
+    RowArgs a = row_args(shape, params, status);
+    a.out = static_cast<uint16_t*>(out_kv_bf16);
+    a.codes = const_cast<uint8_t*>(static_cast<const uint8_t*>(codes));
+    a.scales = const_cast<uint32_t*>(static_cast<const uint32_t*>(scales));
+    bu_maps(shape, z, z.nb * z.pay, z.nb, &a.cmap, &a.smap);
+    cudaError_t e = launch_hadamard(a, false, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "Hadamard decode launch");
+    return CG_OK;
+}
+
 CG_EXPORT int cg_kivi_stream_bytes(const cg_shape* shape, const cg_params* params, size_t* codes_bytes,
                                    size_t* scales_bytes, size_t* ring_bytes, size_t* workspace_bytes) {
     t_err.clear();

@@ -96,6 +96,8 @@ cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_row_move(const MoveArgs& a, cudaStream_t st);
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st);
 cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st);
+// Hadamard gauge by fast Walsh-Hadamard transform (no gauge tensor): encode or decode.
+cudaError_t launch_hadamard(const RowArgs& a, bool encode, cudaStream_t st);
 cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st);
 cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st);
 cudaError_t launch_residual_copy(const ResidArgs& a, cudaStream_t st);

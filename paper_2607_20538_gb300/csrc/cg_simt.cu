@@ -369,6 +369,140 @@ __global__ void __launch_bounds__(kTileWarpsMax * 32) tile_encode_kernel(RowArgs
 }
 
 // ------------------------------------------------------------------------------------
+// Hadamard gauge by fast Walsh-Hadamard transform (the structured Hadamard control of
+// Sec. 4.3, G = H_g / sqrt(g) in fp32 for every (l, s, h, r)), O(g log g) per group and no
+// gauge tensor read. Every entry of G is +-c, c = fp32(1 / sqrt(g)), so the library's
+// products are +-fl(c x_j), and the pairwise summation order over j (adjacent pairs first,
+// halves last) is the butterfly order of the transform (stride 1 first, stride g/2 last):
+// scaling x by c with rounding and then running the butterflies in fp32 gives exactly the
+// library's z. One warp per token row; lane owns CPL = d/32 consecutive channels.
+// ------------------------------------------------------------------------------------
+template <int CPL>
+__device__ __forceinline__ void fwht_lane(float (&v)[CPL], int g, int lane) {
+#pragma unroll
+    for (int h = 1; h < CPL; h <<= 1) {
+        if (h >= g) break;
+#pragma unroll
+        for (int k = 0; k < CPL; k++)
+            if (!(k & h)) {
+                const float a = v[k], b = v[k + h];
+                v[k] = __fadd_rn(a, b);
+                v[k + h] = __fsub_rn(a, b);
+            }
+    }
+    for (int h = CPL; h < g; h <<= 1) {
+        const int m = h / CPL;
+        const bool hi = (lane & m) != 0;
+#pragma unroll
+        for (int k = 0; k < CPL; k++) {
+            const float o = __shfl_xor_sync(0xffffffffu, v[k], m);
+            v[k] = hi ? __fsub_rn(o, v[k]) : __fadd_rn(v[k], o);
+        }
+    }
+}
+
+template <int CPL>
+__global__ void __launch_bounds__(kRowThreads) hadamard_encode_kernel(RowArgs a, float c) {
+    constexpr int d = CPL * 32;
+    __shared__ uint8_t qs_all[kRowWarps][d];
+    __shared__ uint32_t sm_all[kRowWarps][32];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t* qs = qs_all[warp];
+    uint32_t* smw = sm_all[warp];
+    const int g = a.g, bits = a.bits, blk = a.blk, qmax = (1 << bits) - 1;
+    const float qmaxf = (float)qmax;
+    const int lanes_per_blk = blk >= CPL ? blk / CPL : 1;
+    const int nb = d / blk, nw = d * bits / 32;
+    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
+    int32_t flag = 0;
+    for (int64_t row = (int64_t)blockIdx.x * kRowWarps + warp; row < rows; row += (int64_t)gridDim.x * kRowWarps) {
+        const int64_t t = row % a.t_count;
+        int64_t u = row / a.t_count;
+        const int h = (int)(u % a.H); u /= a.H;
+        const int b = (int)(u % a.B); u /= a.B;
+        const int s = a.s_lo + (int)(u % a.s_n);
+        const int l = (int)(u / a.s_n);
+        const uint16_t* xr = a.x + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d + CPL * lane;
+        float v[CPL];
+#pragma unroll
+        for (int k = 0; k < CPL; k++) {
+            const uint32_t xb = xr[k];
+            if (bf16_nonfinite(xb)) flag |= CG_FLAG_NONFINITE_INPUT;
+            v[k] = __fmul_rn(c, bf16_bits_to_float(xb));
+        }
+        fwht_lane<CPL>(v, g, lane);
+        // block ranges: the lane's channels, then the block's lanes
+        float mn = v[0], mx = v[0];
+        if (blk >= CPL) {
+#pragma unroll
+            for (int k = 1; k < CPL; k++) {
+                mn = fminf(mn, v[k]);
+                mx = fmaxf(mx, v[k]);
+            }
+            mn = seg_min(mn, lanes_per_blk);
+            mx = seg_max(mx, lanes_per_blk);
+        }
+#pragma unroll
+        for (int k = 0; k < CPL; k++) {
+            float bmn = mn, bmx = mx;
+            if (blk < CPL) {  // several blocks inside the lane (CPL = 8, block = ... never below 8)
+                const int k0 = (k / blk) * blk;
+                bmn = bmx = v[k0];
+                for (int kk = k0 + 1; kk < k0 + blk; kk++) {
+                    bmn = fminf(bmn, v[kk]);
+                    bmx = fmaxf(bmx, v[kk]);
+                }
+            }
+            const int ch = CPL * lane + k;
+            const uint32_t sz = scale_zero(bmn, bmx, qmaxf, &flag);
+            qs[ch] = (uint8_t)quant_code(v[k], h2f_bits(sz & 0xffffu), h2f_bits(sz >> 16), qmax);
+            if ((ch % blk) == 0) smw[ch / blk] = sz;
+        }
+        __syncwarp();
+        uint32_t* cw = reinterpret_cast<uint32_t*>(a.codes + a.cmap.at(l, s, b, h, t));
+        for (int w = lane; w < nw; w += 32) cw[w] = pack_word(qs, w, bits);
+        if (lane < nb) a.scales[a.smap.at(l, s, b, h, t) + lane] = smw[lane];
+        __syncwarp();
+    }
+    if (flag) raise_flag(a.status, flag);
+}
+
+template <int CPL>
+__global__ void __launch_bounds__(kRowThreads) hadamard_decode_kernel(RowArgs a, float c) {
+    constexpr int d = CPL * 32;
+    __shared__ uint32_t cw_all[kRowWarps][d / 4 + 4];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t* cws = cw_all[warp];
+    const int g = a.g, bits = a.bits, blk = a.blk;
+    const int nw = d * bits / 32;
+    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
+    for (int64_t row = (int64_t)blockIdx.x * kRowWarps + warp; row < rows; row += (int64_t)gridDim.x * kRowWarps) {
+        const int64_t t = row % a.t_count;
+        int64_t u = row / a.t_count;
+        const int h = (int)(u % a.H); u /= a.H;
+        const int b = (int)(u % a.B); u /= a.B;
+        const int s = a.s_lo + (int)(u % a.s_n);
+        const int l = (int)(u / a.s_n);
+        const uint32_t* cw = reinterpret_cast<const uint32_t*>(a.codes + a.cmap.at(l, s, b, h, t));
+        for (int w = lane; w < nw; w += 32) cws[w] = cw[w];
+        __syncwarp();
+        const uint32_t* sp = a.scales + a.smap.at(l, s, b, h, t);
+        float v[CPL];
+#pragma unroll
+        for (int k = 0; k < CPL; k++) {
+            const int ch = CPL * lane + k;
+            const uint32_t sz = __ldg(sp + ch / blk);
+            v[k] = fmaf((float)extract_code(cws, ch * bits, bits), h2f_bits(sz & 0xffffu), h2f_bits(sz >> 16));
+        }
+        fwht_lane<CPL>(v, g, lane);  // H is symmetric: G^T zhat = c H zhat
+        uint16_t* orow = a.out + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d + CPL * lane;
+#pragma unroll
+        for (int k = 0; k < CPL; k++) orow[k] = __bfloat16_as_ushort(__float2bfloat16_rn(c * v[k]));
+        __syncwarp();
+    }
+}
+
+// ------------------------------------------------------------------------------------
 // Row decode: unpack, dequantize zhat = q*s + m, then Xhat = G^T Zhat, bf16 store.
 // ------------------------------------------------------------------------------------
 template <int NR>
@@ -694,6 +828,30 @@ static cudaError_t key_decode_nr(const KeyArgs& a, cudaStream_t st) {
 cudaError_t launch_row_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_encode_nr, a.d, a, st) }
 cudaError_t launch_row_decode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(row_decode_nr, a.d, a, st) }
 cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_SWITCH(tile_encode_nr, a.d, a, st) }
+
+template <int CPL>
+static cudaError_t hadamard_nr(const RowArgs& a, bool enc, cudaStream_t st) {
+    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
+    int64_t grid = (rows + kRowWarps - 1) / kRowWarps;
+    if (grid > 152 * 16) grid = 152 * 16;
+    if (grid < 1) return cudaSuccess;
+    const float c = (float)(1.0 / sqrt((double)a.g));
+    if (enc)
+        hadamard_encode_kernel<CPL><<<(unsigned)grid, kRowThreads, 0, st>>>(a, c);
+    else
+        hadamard_decode_kernel<CPL><<<(unsigned)grid, kRowThreads, 0, st>>>(a, c);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_hadamard(const RowArgs& a, bool encode, cudaStream_t st) {
+    switch (a.d / 32) {
+        case 1: return hadamard_nr<1>(a, encode, st);
+        case 2: return hadamard_nr<2>(a, encode, st);
+        case 4: return hadamard_nr<4>(a, encode, st);
+        case 8: return hadamard_nr<8>(a, encode, st);
+        default: return cudaErrorInvalidValue;
+    }
+}
 cudaError_t launch_key_encode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_encode_nr, a.d, a, st) }
 cudaError_t launch_key_decode_simt(const KeyArgs& a, cudaStream_t st) { CG_NR_SWITCH(key_decode_nr, a.d, a, st) }
 

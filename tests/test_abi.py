@@ -126,6 +126,17 @@ def test_attention_validation(lib):
     assert "workspace" in lib.cg_last_error().decode()
 
 
+def test_hadamard_validation(lib):
+    fake = ctypes.c_void_p(0x10000)
+    S = ctypes.byref(cg.Shape(L=1, B=1, H=1, T=4, d=128).c())
+    for bad in (cg.Params(cg.CG_KIVI, 64, 3, 128, 0), cg.Params(cg.CG_BLOCK_TILE, 64, 4, 64)):
+        assert lib.cg_encode_hadamard(S, ctypes.byref(bad.c()), fake, fake, fake, None) == -2
+        assert lib.cg_decode_hadamard(S, ctypes.byref(bad.c()), fake, fake, fake, None) == -2
+    P = ctypes.byref(cg.Params(0, 64, 4, 64).c())
+    assert lib.cg_encode_hadamard(S, P, None, fake, fake, None) == -1
+    assert lib.cg_encode_hadamard(S, P, ctypes.c_void_p(0x10008), fake, fake, None) == -1
+
+
 def test_pointer_checks_fail_before_device(lib):
     shape = cg.Shape(L=1, B=1, H=1, T=4, d=64)
     params = cg.Params(0, 16, 4, 32)
