@@ -242,22 +242,30 @@ def _setup_cache(w, dev, ws, stream):
     shape, params = cg.Shape(**w.shape), cg.Params(**w.params)
     nc, ns, nr = cg.packed_bytes(shape, params)
     x = synth.kv_cache(w, threads=max(4, (os.cpu_count() or 8) // max(ws, 1)))
-    P.G = synth.gauges(w)
+    hadamard = w.extra.get("gauge") == "hadamard"
+    P.G = synth.gauges(w, "hadamard" if hadamard else "random")
     dx = torch.from_numpy(x.reshape(-1).view(np.int16)).to(dev)
     dG = torch.from_numpy(P.G.reshape(-1)).to(dev)
     codes, scales, resid = cg.alloc_outputs(shape, params, device=dev)
     out = torch.empty_like(dx)
     n = x.nbytes
     P.enc_bytes = P.dec_bytes = n
-    P.enc_alg = P.dec_alg = n + nc + ns + nr + P.G.nbytes
+    P.enc_alg = P.dec_alg = n + nc + ns + nr + (0 if hadamard else P.G.nbytes)
     P.launches = 2 if w.backend != 1 else 2 * 3
-    P.config = {}
+    P.config = {"gauge": "hadamard by fast Walsh-Hadamard transform (no gauge tensor)"} if hadamard else {}
 
-    def encode():
-        cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+    if hadamard:
+        def encode():
+            cg.encode_hadamard(shape, params, dx, codes, scales, stream=stream)
 
-    def decode():
-        cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
+        def decode():
+            cg.decode_hadamard(shape, params, codes, scales, out, stream=stream)
+    else:
+        def encode():
+            cg.encode(shape, params, dx, dG, codes, scales, resid, stream=stream)
+
+        def decode():
+            cg.decode(shape, params, codes, scales, resid, dG, out, stream=stream)
 
     P.encode, P.decode = encode, decode
     hx = torch.from_numpy(x.reshape(-1).view(np.int16)).pin_memory()
@@ -286,8 +294,12 @@ def _setup_cache(w, dev, ws, stream):
             c1 = codes[l * nc1:(l + 1) * nc1]
             sc1 = scales[l * (ns1 // 4):(l + 1) * (ns1 // 4)]
             r1 = resid[l * (nr1 // 2):(l + 1) * (nr1 // 2)] if nr1 else None
-            cg.encode(shape1, params, dx[xs], dG[gs], c1, sc1, r1, stream=stream)
-            cg.decode(shape1, params, c1, sc1, r1, dG[gs], out[xs], stream=stream)
+            if hadamard:
+                cg.encode_hadamard(shape1, params, dx[xs], c1, sc1, stream=stream)
+                cg.decode_hadamard(shape1, params, c1, sc1, out[xs], stream=stream)
+            else:
+                cg.encode(shape1, params, dx[xs], dG[gs], c1, sc1, r1, stream=stream)
+                cg.decode(shape1, params, c1, sc1, r1, dG[gs], out[xs], stream=stream)
             ev_done[l].record(stream)
             s_out.wait_event(ev_done[l])
             with torch.cuda.stream(s_out):
@@ -537,7 +549,8 @@ PAPER_CONTEXT = {
 }
 
 # The other target workloads, timed in the same process after the headline one.
-EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "rolling_attn", "kivi3_stream", "llama3_8b_tile")
+EXTRA_WORKLOADS = ("gemma27b", "kivi3_qwen", "rolling", "rolling_attn", "kivi3_stream", "llama3_8b_tile",
+                   "llama3_8b_hadamard")
 
 
 def run_cuda(args):

@@ -401,6 +401,41 @@ __device__ __forceinline__ void fwht_lane(float (&v)[CPL], int g, int lane) {
     }
 }
 
+// CPL consecutive bf16 values (CPL * 2 bytes, naturally aligned) as raw bits.
+template <int CPL>
+__device__ __forceinline__ void load_bf16(const uint16_t* p, uint32_t (&out)[CPL]) {
+    if (CPL == 8) {
+        const uint4 v = *reinterpret_cast<const uint4*>(p);
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < CPL; k++) out[k] = (w[k >> 1] >> (16 * (k & 1))) & 0xffffu;
+    } else if (CPL == 4) {
+        const uint2 v = *reinterpret_cast<const uint2*>(p);
+        const uint32_t w[2] = {v.x, v.y};
+#pragma unroll
+        for (int k = 0; k < CPL; k++) out[k] = (w[k >> 1] >> (16 * (k & 1))) & 0xffffu;
+    } else if (CPL == 2) {
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
+        out[0] = w & 0xffffu;
+        out[CPL - 1] = w >> 16;
+    } else {
+        out[0] = p[0];
+    }
+}
+
+// The rule's code, clamp(rint(fl((z - m) / s)), 0, qmax), from a reciprocal product: the product
+// is within a few ulp of the quotient, so it rounds to the same integer unless it lies within
+// 2^-12 of a half-integer, where the exact division decides (rare).
+__device__ __forceinline__ uint32_t quant_code_rcp(float z, float s, float m, float rcp, int qmax) {
+    if (s == 0.0f) return 0u;
+    const float d = __fsub_rn(z, m);
+    float t = __fmul_rn(d, rcp);
+    if (fabsf(t - floorf(t) - 0.5f) < 2.5e-4f) t = __fdiv_rn(d, s);
+    int q = __float2int_rn(t);
+    q = q < 0 ? 0 : (q > qmax ? qmax : q);
+    return (uint32_t)q;
+}
+
 template <int CPL>
 __global__ void __launch_bounds__(kRowThreads) hadamard_encode_kernel(RowArgs a, float c) {
     constexpr int d = CPL * 32;
@@ -411,57 +446,49 @@ __global__ void __launch_bounds__(kRowThreads) hadamard_encode_kernel(RowArgs a,
     uint32_t* smw = sm_all[warp];
     const int g = a.g, bits = a.bits, blk = a.blk, qmax = (1 << bits) - 1;
     const float qmaxf = (float)qmax;
-    const int lanes_per_blk = blk >= CPL ? blk / CPL : 1;
+    const int lanes_per_blk = blk / CPL;  // block >= 8 >= CPL
     const int nb = d / blk, nw = d * bits / 32;
-    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
+    // grid: x = (l, s, b, h) unit, y = token range; a warp takes tokens in steps of the y extent
+    int u = blockIdx.x;
+    const int h = u % a.H; u /= a.H;
+    const int b = u % a.B; u /= a.B;
+    const int s = a.s_lo + u % a.s_n;
+    const int l = u / a.s_n;
+    const uint16_t* xu = a.x + (((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x * d + CPL * lane;
+    const int64_t stride = (int64_t)gridDim.y * kRowWarps;
     int32_t flag = 0;
-    for (int64_t row = (int64_t)blockIdx.x * kRowWarps + warp; row < rows; row += (int64_t)gridDim.x * kRowWarps) {
-        const int64_t t = row % a.t_count;
-        int64_t u = row / a.t_count;
-        const int h = (int)(u % a.H); u /= a.H;
-        const int b = (int)(u % a.B); u /= a.B;
-        const int s = a.s_lo + (int)(u % a.s_n);
-        const int l = (int)(u / a.s_n);
-        const uint16_t* xr = a.x + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d + CPL * lane;
+    int64_t t = (int64_t)blockIdx.y * kRowWarps + warp;
+    uint32_t xb[CPL];
+    if (t < a.t_count) load_bf16<CPL>(xu + t * d, xb);
+    for (; t < a.t_count; t += stride) {
         float v[CPL];
 #pragma unroll
         for (int k = 0; k < CPL; k++) {
-            const uint32_t xb = xr[k];
-            if (bf16_nonfinite(xb)) flag |= CG_FLAG_NONFINITE_INPUT;
-            v[k] = __fmul_rn(c, bf16_bits_to_float(xb));
+            if (bf16_nonfinite(xb[k])) flag |= CG_FLAG_NONFINITE_INPUT;
+            v[k] = __fmul_rn(c, bf16_bits_to_float(xb[k]));
         }
+        const int cl = l, cs = s, cb = b, ch_ = h;
+        const int64_t ct = t;
+        if (t + stride < a.t_count) load_bf16<CPL>(xu + (t + stride) * d, xb);  // next row
         fwht_lane<CPL>(v, g, lane);
-        // block ranges: the lane's channels, then the block's lanes
         float mn = v[0], mx = v[0];
-        if (blk >= CPL) {
 #pragma unroll
-            for (int k = 1; k < CPL; k++) {
-                mn = fminf(mn, v[k]);
-                mx = fmaxf(mx, v[k]);
-            }
-            mn = seg_min(mn, lanes_per_blk);
-            mx = seg_max(mx, lanes_per_blk);
+        for (int k = 1; k < CPL; k++) {
+            mn = fminf(mn, v[k]);
+            mx = fmaxf(mx, v[k]);
         }
+        mn = seg_min(mn, lanes_per_blk);
+        mx = seg_max(mx, lanes_per_blk);
+        const uint32_t sz = scale_zero(mn, mx, qmaxf, &flag);
+        const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
+        const float rcp = sc != 0.0f ? __frcp_rn(sc) : 0.0f;
 #pragma unroll
-        for (int k = 0; k < CPL; k++) {
-            float bmn = mn, bmx = mx;
-            if (blk < CPL) {  // several blocks inside the lane (CPL = 8, block = ... never below 8)
-                const int k0 = (k / blk) * blk;
-                bmn = bmx = v[k0];
-                for (int kk = k0 + 1; kk < k0 + blk; kk++) {
-                    bmn = fminf(bmn, v[kk]);
-                    bmx = fmaxf(bmx, v[kk]);
-                }
-            }
-            const int ch = CPL * lane + k;
-            const uint32_t sz = scale_zero(bmn, bmx, qmaxf, &flag);
-            qs[ch] = (uint8_t)quant_code(v[k], h2f_bits(sz & 0xffffu), h2f_bits(sz >> 16), qmax);
-            if ((ch % blk) == 0) smw[ch / blk] = sz;
-        }
+        for (int k = 0; k < CPL; k++) qs[CPL * lane + k] = (uint8_t)quant_code_rcp(v[k], sc, mz, rcp, qmax);
+        if (((CPL * lane) % blk) == 0) smw[(CPL * lane) / blk] = sz;
         __syncwarp();
-        uint32_t* cw = reinterpret_cast<uint32_t*>(a.codes + a.cmap.at(l, s, b, h, t));
+        uint32_t* cw = reinterpret_cast<uint32_t*>(a.codes + a.cmap.at(cl, cs, cb, ch_, ct));
         for (int w = lane; w < nw; w += 32) cw[w] = pack_word(qs, w, bits);
-        if (lane < nb) a.scales[a.smap.at(l, s, b, h, t) + lane] = smw[lane];
+        if (lane < nb) a.scales[a.smap.at(cl, cs, cb, ch_, ct) + lane] = smw[lane];
         __syncwarp();
     }
     if (flag) raise_flag(a.status, flag);
@@ -470,35 +497,44 @@ __global__ void __launch_bounds__(kRowThreads) hadamard_encode_kernel(RowArgs a,
 template <int CPL>
 __global__ void __launch_bounds__(kRowThreads) hadamard_decode_kernel(RowArgs a, float c) {
     constexpr int d = CPL * 32;
-    __shared__ uint32_t cw_all[kRowWarps][d / 4 + 4];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    uint32_t* cws = cw_all[warp];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = a.g, bits = a.bits, blk = a.blk;
     const int nw = d * bits / 32;
-    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
-    for (int64_t row = (int64_t)blockIdx.x * kRowWarps + warp; row < rows; row += (int64_t)gridDim.x * kRowWarps) {
-        const int64_t t = row % a.t_count;
-        int64_t u = row / a.t_count;
-        const int h = (int)(u % a.H); u /= a.H;
-        const int b = (int)(u % a.B); u /= a.B;
-        const int s = a.s_lo + (int)(u % a.s_n);
-        const int l = (int)(u / a.s_n);
+    const uint32_t mask = (1u << bits) - 1u;
+    const int bit0 = CPL * lane * bits, wi = bit0 >> 5, sh = bit0 & 31;
+    int u = blockIdx.x;  // grid as in the encode kernel
+    const int h = u % a.H; u /= a.H;
+    const int b = u % a.B; u /= a.B;
+    const int s = a.s_lo + u % a.s_n;
+    const int l = u / a.s_n;
+    for (int64_t t = (int64_t)blockIdx.y * kRowWarps + warp; t < a.t_count; t += (int64_t)gridDim.y * kRowWarps) {
+        // this lane's CPL codes: CPL * bits <= 64 bits starting at bit bit0 of the row
         const uint32_t* cw = reinterpret_cast<const uint32_t*>(a.codes + a.cmap.at(l, s, b, h, t));
-        for (int w = lane; w < nw; w += 32) cws[w] = cw[w];
-        __syncwarp();
-        const uint32_t* sp = a.scales + a.smap.at(l, s, b, h, t);
+        const uint32_t w0 = __ldg(cw + wi);
+        const uint32_t w1 = wi + 1 < nw ? __ldg(cw + wi + 1) : 0u;
+        const uint32_t w2 = wi + 2 < nw ? __ldg(cw + wi + 2) : 0u;
+        const uint64_t lo = (((uint64_t)w1 << 32) | w0) >> sh;
+        const uint64_t cv = sh ? (lo | ((uint64_t)w2 << (64 - sh))) : lo;
+        const uint32_t sz = __ldg(a.scales + a.smap.at(l, s, b, h, t) + (CPL * lane) / blk);
+        const float sc = h2f_bits(sz & 0xffffu), mz = h2f_bits(sz >> 16);
         float v[CPL];
 #pragma unroll
-        for (int k = 0; k < CPL; k++) {
-            const int ch = CPL * lane + k;
-            const uint32_t sz = __ldg(sp + ch / blk);
-            v[k] = fmaf((float)extract_code(cws, ch * bits, bits), h2f_bits(sz & 0xffffu), h2f_bits(sz >> 16));
-        }
+        for (int k = 0; k < CPL; k++) v[k] = fmaf((float)((uint32_t)(cv >> (k * bits)) & mask), sc, mz);
         fwht_lane<CPL>(v, g, lane);  // H is symmetric: G^T zhat = c H zhat
         uint16_t* orow = a.out + ((((int64_t)(l * 2 + s) * a.B + b) * a.H + h) * a.T_x + t) * d + CPL * lane;
+        uint32_t ob[CPL];
 #pragma unroll
-        for (int k = 0; k < CPL; k++) orow[k] = __bfloat16_as_ushort(__float2bfloat16_rn(c * v[k]));
-        __syncwarp();
+        for (int k = 0; k < CPL; k++) ob[k] = __bfloat16_as_ushort(__float2bfloat16_rn(c * v[k]));
+        if (CPL == 8) {
+            *reinterpret_cast<uint4*>(orow) = make_uint4(ob[0] | ob[1 % CPL] << 16, ob[2 % CPL] | ob[3 % CPL] << 16,
+                                                         ob[4 % CPL] | ob[5 % CPL] << 16, ob[6 % CPL] | ob[7 % CPL] << 16);
+        } else if (CPL == 4) {
+            *reinterpret_cast<uint2*>(orow) = make_uint2(ob[0] | ob[1 % CPL] << 16, ob[2 % CPL] | ob[3 % CPL] << 16);
+        } else if (CPL == 2) {
+            *reinterpret_cast<uint32_t*>(orow) = ob[0] | ob[1 % CPL] << 16;
+        } else {
+            orow[0] = (uint16_t)ob[0];
+        }
     }
 }
 
@@ -831,15 +867,17 @@ cudaError_t launch_tile_encode_simt(const RowArgs& a, cudaStream_t st) { CG_NR_S
 
 template <int CPL>
 static cudaError_t hadamard_nr(const RowArgs& a, bool enc, cudaStream_t st) {
-    const int64_t rows = (int64_t)a.L * a.s_n * a.B * a.H * a.t_count;
-    int64_t grid = (rows + kRowWarps - 1) / kRowWarps;
-    if (grid > 152 * 16) grid = 152 * 16;
-    if (grid < 1) return cudaSuccess;
+    const int64_t units = (int64_t)a.L * a.s_n * a.B * a.H;
+    if (units < 1 || a.t_count < 1) return cudaSuccess;
+    // token ranges per unit: about 8 rows per warp, at most 65535 ranges
+    int64_t gy = (a.t_count + 8 * kRowWarps - 1) / (8 * kRowWarps);
+    if (gy > 65535) gy = 65535;
+    const dim3 grid((unsigned)units, (unsigned)gy);
     const float c = (float)(1.0 / sqrt((double)a.g));
     if (enc)
-        hadamard_encode_kernel<CPL><<<(unsigned)grid, kRowThreads, 0, st>>>(a, c);
+        hadamard_encode_kernel<CPL><<<grid, kRowThreads, 0, st>>>(a, c);
     else
-        hadamard_decode_kernel<CPL><<<(unsigned)grid, kRowThreads, 0, st>>>(a, c);
+        hadamard_decode_kernel<CPL><<<grid, kRowThreads, 0, st>>>(a, c);
     return cudaGetLastError();
 }
 

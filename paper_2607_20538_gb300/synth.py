@@ -93,6 +93,10 @@ WORKLOADS = {
     "kivi3_stream": Workload("kivi3_stream", L=28, B=4, H=4, T=32768, d=128, group=64, backend=1, bits=3,
                              block=128, residual=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,
                              kv_seed=1002, gauge_seed=2002, T_cap=32768),
+    # the 8B cache under the Hadamard gauge, applied by fast Walsh-Hadamard transform
+    "llama3_8b_hadamard": Workload("llama3_8b_hadamard", L=32, B=1, H=8, T=8192, d=128, group=128, backend=0,
+                                   bits=4, block=64, n_outlier=4, outlier_mult=10.0, sigma_v=0.3, kv_seed=1001,
+                                   gauge_seed=2001, extra={"gauge": "hadamard"}),
     # the paper's block-uniform block shape on the 8B cache: one range per 16-token x d tile
     "llama3_8b_tile": Workload("llama3_8b_tile", L=32, B=1, H=8, T=8192, d=128, group=128, backend=3,
                                bits=4, block=128, n_outlier=4, outlier_mult=10.0, sigma_v=0.3,
