@@ -15,7 +15,7 @@
 //
 // Kernels: attn_query_kernel (q' = scale * G_K q); a chunk kernel that writes, per (l, b, h) and
 // part, the part's softmax max, sum and gauge-space weighted value sum (attn_chunk_mma_kernel for
-// 2- and 4-bit codes: many 256-token chunks per CTA, codes staged by bulk copies one chunk ahead,
+// 2- and 4-bit codes: many 128-token chunks per CTA, codes staged by bulk copies one chunk ahead,
 // online softmax; attn_chunk_kernel for 3-, 6- and 8-bit codes: one chunk per CTA, all on CUDA
 // cores); attn_combine_kernel (merges the parts, applies G_V^T).
 #include "cg_launch.h"
@@ -359,17 +359,19 @@ struct MmaSmem {
     static constexpr int run = c32 + NREP * 4 * 4;                    // [NREP] max, sum, alpha; [NREP][4] W, Z
     static constexpr int scratch = run + NREP * (3 + 8) * 4;          // [4 warps][NREP * 4]
     static constexpr int outv = scratch + 4 * NREP * 4 * 4;           // [NREP * 4] reduction results
-    static constexpr int sv = outv + NREP * 4 * 4;                    // [chunk][4] value scales
-    static constexpr int p = sv + kAttnChunk * 4 * 4;                 // [NREP][chunk] scores / p; red
+    static constexpr int sk = outv + NREP * 4 * 4;                    // [2][chunk][4] key scales
+    static constexpr int sv = sk + 2 * kAttnChunk * 4 * 4;            // [2][chunk][4] value scales
+    static constexpr int p = sv + 2 * kAttnChunk * 4 * 4;             // [NREP][chunk] scores / p; red
     static constexpr int pbytes = NREP * kAttnChunk * 4, rbytes = (kMThreads / 16) * NREP * kAD * 4;
     static constexpr int total = p + (pbytes > rbytes ? pbytes : rbytes);
 };
 
-// One CTA per (l, b, h) and part: the part's 256-token chunks in order, the next chunk's key
-// and value codes arriving by bulk copy into the other stage while this one is computed, and
-// an online softmax over the chunks (running max; earlier sums rescaled by exp(old - new)).
+// One CTA per (l, b, h) and part: the part's chunks in order, the next chunk's key and value
+// codes arriving by bulk copy into the other stage (and its scales by loads held in registers)
+// while this one is computed, and an online softmax over the chunks (running max; earlier sums
+// rescaled by exp(old - new); each thread keeps its own sums until the end).
 template <int BITS, int NREP>
-__global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
+__global__ void __launch_bounds__(kMThreads, 3) attn_chunk_mma_kernel(AttnArgs a) {
     static_assert(BITS == 2 || BITS == 4, "tensor-core attention serves 2- and 4-bit codes");
     using SL = MmaSmem<BITS, NREP>;
     constexpr int kWords = kAD * BITS / 32;  // code words per token row
@@ -386,7 +388,8 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
     float* Wr = alpha + NREP;   // [NREP][4]
     float* Zr = Wr + NREP * 4;  // [NREP][4]
     float* scratch = reinterpret_cast<float*>(smem + SL::scratch);
-    uint32_t* SV = reinterpret_cast<uint32_t*>(smem + SL::sv);
+    uint32_t* SKb = reinterpret_cast<uint32_t*>(smem + SL::sk);
+    uint32_t* SVb = reinterpret_cast<uint32_t*>(smem + SL::sv);
     float* P = reinterpret_cast<float*>(smem + SL::p);
     float* outv = reinterpret_cast<float*>(smem + SL::outv);
 
@@ -411,18 +414,53 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
                   &bars[2 * st + 1]);
     };
 
+    // the key and value scales of a chunk's tokens: tokens tid, tid + 128, ... of the chunk
+    auto load_scales = [&](int ci, uint32_t (&ks)[kAttnChunk / kMThreads][4], uint32_t (&vs)[kAttnChunk / kMThreads][4]) {
+        const int64_t c0 = (int64_t)ci * kAttnChunk;
+        const int n = chunk_tokens(ci);
+#pragma unroll
+        for (int q = 0; q < kAttnChunk / kMThreads; q++) {
+            const int tt = tid + q * kMThreads;
+#pragma unroll
+            for (int k = 0; k < 4; k++) ks[q][k] = vs[q][k] = 0u;
+            if (tt < n) {
+                const uint32_t* kp = a.scales + a.smap.at(l, 0, b, h, c0 + tt);
+                const uint32_t* vp = a.scales + a.smap.at(l, 1, b, h, c0 + tt);
+#pragma unroll
+                for (int k = 0; k < 4; k++)
+                    if (k < nb) {
+                        ks[q][k] = __ldg(kp + k);
+                        vs[q][k] = __ldg(vp + k);
+                    }
+            }
+        }
+    };
+    auto store_scales = [&](int bufi, const uint32_t (&ks)[kAttnChunk / kMThreads][4],
+                            const uint32_t (&vs)[kAttnChunk / kMThreads][4]) {
+#pragma unroll
+        for (int q = 0; q < kAttnChunk / kMThreads; q++) {
+            const int tt = tid + q * kMThreads;
+#pragma unroll
+            for (int k = 0; k < 4; k++) {
+                SKb[(bufi * kAttnChunk + tt) * 4 + k] = ks[q][k];
+                SVb[(bufi * kAttnChunk + tt) * 4 + k] = vs[q][k];
+            }
+        }
+    };
+    uint32_t nks[kAttnChunk / kMThreads][4], nvs[kAttnChunk / kMThreads][4];
+
     if (tid == 0) {
         abort_flag[0] = 0;
         abort_flag[1] = 0;
         for (int k = 0; k < 4; k++) mbar_init(&bars[k], 1);
         fence_barrier_init();
     }
-    for (int e = tid; e < NREP * kAD; e += kMThreads) qs[e] = a.qrot[(int64_t)unit * NREP * kAD + e];
-    if (tid < NREP) {
-        Mrun[tid] = -INFINITY;
-        Lrun[tid] = 0.0f;
+    if (ch_lo < ch_hi) {
+        load_scales(ch_lo, nks, nvs);
+        store_scales(0, nks, nvs);
     }
-    if (tid < NREP * 4) Wr[tid] = Zr[tid] = 0.0f;
+    for (int e = tid; e < NREP * kAD; e += kMThreads) qs[e] = a.qrot[(int64_t)unit * NREP * kAD + e];
+    if (tid < NREP) Mrun[tid] = -INFINITY;
     __syncthreads();
     if (tid == 0 && ch_lo < ch_hi) issue(ch_lo, 0);
     if (tid < NREP * 4) {
@@ -450,10 +488,21 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
     for (int r = 0; r < NREP; r++)
 #pragma unroll
         for (int k = 0; k < 8; k++) acc[r][k] = 0.0f;
+    // this thread's share of the softmax sums: sum p, sum p s_V and sum p m_V per block
+    float lsum[NREP], wsum[NREP][4], zsum[NREP][4];
+#pragma unroll
+    for (int r = 0; r < NREP; r++) {
+        lsum[r] = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 4; k++) wsum[r][k] = zsum[r][k] = 0.0f;
+    }
 
     for (int ci = ch_lo; ci < ch_hi; ci++) {
         const int it = ci - ch_lo, st = it & 1;
         const uint32_t par = (uint32_t)(it >> 1) & 1u;
+        const uint32_t* SK = SKb + st * kAttnChunk * 4;
+        const uint32_t* SV = SVb + st * kAttnChunk * 4;
+        if (ci + 1 < ch_hi) load_scales(ci + 1, nks, nvs);  // stored after this chunk
         const unsigned char* Kc = smem + SL::codes + (2 * st) * SL::kStage;
         const unsigned char* Vc = Kc + SL::kStage;
         const int64_t c0 = (int64_t)ci * kAttnChunk;
@@ -516,10 +565,9 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
             for (int half = 0; half < 2; half++) {
                 const int r = half ? r1 : r0;
                 if (r >= n_tok) continue;
-                const uint32_t* sk = a.scales + a.smap.at(l, 0, b, h, c0 + r);
                 uint32_t sz[4];
 #pragma unroll
-                for (int k = 0; k < 4; k++) sz[k] = k < nb ? __ldg(sk + k) : 0u;
+                for (int k = 0; k < 4; k++) sz[k] = SK[r * 4 + k];
 #pragma unroll
                 for (int cq = 0; cq < 2; cq++) {
                     const int q = 2 * t + cq;
@@ -552,54 +600,36 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
                 Mrun[tid] = mn;
             }
             __syncthreads();
-            float ws[NREP * 4], zs[NREP * 4], es[NREP];
 #pragma unroll
-            for (int k = 0; k < NREP * 4; k++) ws[k] = zs[k] = 0.0f;
-#pragma unroll
-            for (int r = 0; r < NREP; r++) es[r] = 0.0f;
-            for (int tt = tid; tt < ngrp * 16; tt += kMThreads) {
-                if (tt >= n_tok) {  // padding tokens of the last group: weight 0
-#pragma unroll
-                    for (int r = 0; r < NREP; r++) P[r * kAttnChunk + tt] = 0.0f;
-#pragma unroll
-                    for (int k = 0; k < 4; k++) SV[tt * 4 + k] = 0u;
-                    continue;
-                }
-                const uint32_t* svp = a.scales + a.smap.at(l, 1, b, h, c0 + tt);
-                uint32_t z[4];
+            for (int r = 0; r < NREP; r++) {
+                const float al = alpha[r];
+                lsum[r] *= al;
 #pragma unroll
                 for (int k = 0; k < 4; k++) {
-                    z[k] = k < nb ? __ldg(svp + k) : 0u;
-                    SV[tt * 4 + k] = z[k];
+                    wsum[r][k] *= al;
+                    zsum[r][k] *= al;
                 }
+#pragma unroll
+                for (int k = 0; k < 8; k++) acc[r][k] *= al;
+            }
+            for (int tt = tid; tt < n_tok; tt += kMThreads) {
+                uint32_t z[4];
+#pragma unroll
+                for (int k = 0; k < 4; k++) z[k] = SV[tt * 4 + k];
 #pragma unroll
                 for (int r = 0; r < NREP; r++) {
                     const float p = __expf(P[r * kAttnChunk + tt] - Mrun[r]);
                     P[r * kAttnChunk + tt] = p;
-                    es[r] += p;
+                    lsum[r] += p;
 #pragma unroll
                     for (int k = 0; k < 4; k++) {
-                        ws[r * 4 + k] = fmaf(p, half_lo(z[k]), ws[r * 4 + k]);
-                        zs[r * 4 + k] = fmaf(p, half_hi(z[k]), zs[r * 4 + k]);
+                        wsum[r][k] = fmaf(p, half_lo(z[k]), wsum[r][k]);
+                        zsum[r][k] = fmaf(p, half_hi(z[k]), zsum[r][k]);
                     }
                 }
             }
-            block_reduce_n<NREP, false, kMThreads>(es, scratch, outv);
-            if (tid < NREP) Lrun[tid] = Lrun[tid] * alpha[tid] + outv[tid];
-            __syncthreads();
-            block_reduce_n<NREP * 4, false, kMThreads>(ws, scratch, outv);
-            if (tid < NREP * 4) Wr[tid] = Wr[tid] * alpha[tid >> 2] + outv[tid];
-            __syncthreads();
-            block_reduce_n<NREP * 4, false, kMThreads>(zs, scratch, outv);
-            if (tid < NREP * 4) Zr[tid] = Zr[tid] * alpha[tid >> 2] + outv[tid];
         }
-        {
-            // rescale this thread's value sums to the new running max
-#pragma unroll
-            for (int r = 0; r < NREP; r++)
-#pragma unroll
-                for (int k = 0; k < 8; k++) acc[r][k] *= alpha[r];
-        }
+        __syncthreads();
 
         // values on CUDA cores: thread = 8 channels (one 32-bit group of 4-bit codes, half of
         // one for 2-bit) x token slice; sum_t (p s_V) f per channel, f = 1 + q 2^-b
@@ -629,7 +659,29 @@ __global__ void __launch_bounds__(kMThreads) attn_chunk_mma_kernel(AttnArgs a) {
                 }
             }
         }
-        __syncthreads();  // P, SV and this stage's codes are free for the next chunk
+        __syncthreads();  // P, the scales and this stage's codes are free for the next chunk
+        if (ci + 1 < ch_hi) store_scales(st ^ 1, nks, nvs);
+    }
+    // the sums over threads (one reduction of each, after the last chunk)
+    block_reduce_n<NREP, false, kMThreads>(lsum, scratch, outv);
+    if (tid < NREP) Lrun[tid] = outv[tid];
+    __syncthreads();
+    {
+        float wv[NREP * 4];
+#pragma unroll
+        for (int r = 0; r < NREP; r++)
+#pragma unroll
+            for (int k = 0; k < 4; k++) wv[r * 4 + k] = wsum[r][k];
+        block_reduce_n<NREP * 4, false, kMThreads>(wv, scratch, outv);
+        if (tid < NREP * 4) Wr[tid] = outv[tid];
+        __syncthreads();
+#pragma unroll
+        for (int r = 0; r < NREP; r++)
+#pragma unroll
+            for (int k = 0; k < 4; k++) wv[r * 4 + k] = zsum[r][k];
+        block_reduce_n<NREP * 4, false, kMThreads>(wv, scratch, outv);
+        if (tid < NREP * 4) Zr[tid] = outv[tid];
+        __syncthreads();
     }
 
     // the slices' sums, then the sum over slices (red reuses P's space)

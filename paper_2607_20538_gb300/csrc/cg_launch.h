@@ -85,7 +85,7 @@ struct AttnArgs {
     uint64_t wait_ns;       // limit of the bounded waits on the chunk copies
 };
 
-constexpr int kAttnChunk = 256;  // tokens per CTA of the chunk kernels
+constexpr int kAttnChunk = 128;  // tokens per chunk of the chunk kernels
 size_t attn_workspace_bytes(int64_t units, int n_rep, int d, int64_t T);
 cudaError_t launch_attention(const AttnArgs& a, cudaStream_t st);
 

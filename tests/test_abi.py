@@ -111,7 +111,7 @@ def test_attention_validation(lib):
     """cg_attention: supported caches and query-head counts are checked on the host."""
     sh = cg.Shape(L=2, B=3, H=2, T=1100, d=128)
     nb = cg.attention_workspace_bytes(sh, cg.Params(0, 128, 4, 64), 4)
-    assert nb == -(-2 * 3 * 2 * 4 * 128 * 4 // 256) * 256 + 2 * 3 * 2 * 5 * 4 * 130 * 4   # queries, 5 chunks
+    assert nb == -(-2 * 3 * 2 * 4 * 128 * 4 // 256) * 256 + 2 * 3 * 2 * 9 * 4 * 130 * 4   # queries, 9 chunks
     for params, n_rep in ((cg.Params(cg.CG_KIVI, 64, 3, 128, 128), 4), (cg.Params(0, 16, 4, 16), 4),
                           (cg.Params(0, 16, 4, 64), 3)):
         with pytest.raises(cg.CodecGaugeError):
