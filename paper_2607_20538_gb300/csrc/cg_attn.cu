@@ -324,6 +324,14 @@ __device__ __forceinline__ uint32_t pair_bf16(uint32_t x) {
     return ((x * kMul) & kMask) | kOne;
 }
 
+// (d0, d1) += a * (b0, b1): one packed fp32 fused multiply-add (each lane rounded once, as fmaf).
+__device__ __forceinline__ void ffma2(float& d0, float& d1, float a, float b0, float b1) {
+    asm("{\n\t.reg .b64 dd, aa, bb;\n\tmov.b64 dd, {%0, %1};\n\tmov.b64 aa, {%2, %2};\n\t"
+        "mov.b64 bb, {%3, %4};\n\tfma.rn.f32x2 dd, aa, bb, dd;\n\tmov.b64 {%0, %1}, dd;\n\t}"
+        : "+f"(d0), "+f"(d1)
+        : "f"(a), "f"(b0), "f"(b1));
+}
+
 // v[i] for a runtime i < 4 without indexing a register array (no local memory).
 template <typename T>
 __device__ __forceinline__ T pick4(const T (&v)[4], int i) {
@@ -361,7 +369,7 @@ struct MmaSmem {
     static constexpr int outv = scratch + 4 * NREP * 4 * 4;           // [NREP * 4] reduction results
     static constexpr int sk = outv + NREP * 4 * 4;                    // [2][chunk][4] key scales
     static constexpr int sv = sk + 2 * kAttnChunk * 4 * 4;            // [2][chunk][4] value scales
-    static constexpr int p = sv + 2 * kAttnChunk * 4 * 4;             // [NREP][chunk] scores / p; red
+    static constexpr int p = sv + 2 * kAttnChunk * 4 * 4;             // [chunk][NREP] scores / p; red
     static constexpr int pbytes = NREP * kAttnChunk * 4, rbytes = (kMThreads / 16) * NREP * kAD * 4;
     static constexpr int total = p + (pbytes > rbytes ? pbytes : rbytes);
 };
@@ -579,7 +587,7 @@ __global__ void __launch_bounds__(kMThreads, 3) attn_chunk_mma_kernel(AttnArgs a
                         const float sc = half_lo(z), mz = half_hi(z);
                         s += sc * d[k][2 * half + cq] + (mz - kOff * sc) * c32[q * 4 + k];
                     }
-                    P[q * kAttnChunk + r] = s;
+                    P[r * NREP + q] = s;
                 }
             }
         }
@@ -591,7 +599,7 @@ __global__ void __launch_bounds__(kMThreads, 3) attn_chunk_mma_kernel(AttnArgs a
 #pragma unroll
             for (int r = 0; r < NREP; r++) {
                 v[r] = -INFINITY;
-                for (int tt = tid; tt < n_tok; tt += kMThreads) v[r] = fmaxf(v[r], P[r * kAttnChunk + tt]);
+                for (int tt = tid; tt < n_tok; tt += kMThreads) v[r] = fmaxf(v[r], P[tt * NREP + r]);
             }
             block_reduce_n<NREP, true, kMThreads>(v, scratch, outv);
             if (tid < NREP) {
@@ -618,8 +626,8 @@ __global__ void __launch_bounds__(kMThreads, 3) attn_chunk_mma_kernel(AttnArgs a
                 for (int k = 0; k < 4; k++) z[k] = SV[tt * 4 + k];
 #pragma unroll
                 for (int r = 0; r < NREP; r++) {
-                    const float p = __expf(P[r * kAttnChunk + tt] - Mrun[r]);
-                    P[r * kAttnChunk + tt] = p;
+                    const float p = __expf(P[tt * NREP + r] - Mrun[r]);
+                    P[tt * NREP + r] = p;
                     lsum[r] += p;
 #pragma unroll
                     for (int k = 0; k < 4; k++) {
@@ -650,13 +658,15 @@ __global__ void __launch_bounds__(kMThreads, 3) attn_chunk_mma_kernel(AttnArgs a
                 const float s_v = half_lo(SV[tt * 4 + vbk]);
                 float wgt[NREP];
 #pragma unroll
-                for (int r = 0; r < NREP; r++) wgt[r] = P[r * kAttnChunk + tt] * s_v;
+                for (int r = 0; r < NREP; r++) wgt[r] = P[tt * NREP + r] * s_v;
+                float f[8];
 #pragma unroll
-                for (int k = 0; k < 8; k++) {
-                    const float f = __uint_as_float(0x3F800000u | (((bits >> (k * BITS)) & ((1u << BITS) - 1u)) << (23 - BITS)));
+                for (int k = 0; k < 8; k++)
+                    f[k] = __uint_as_float(0x3F800000u | (((bits >> (k * BITS)) & ((1u << BITS) - 1u)) << (23 - BITS)));
 #pragma unroll
-                    for (int r = 0; r < NREP; r++) acc[r][k] = fmaf(wgt[r], f, acc[r][k]);
-                }
+                for (int r = 0; r < NREP; r++)
+#pragma unroll
+                    for (int k = 0; k < 8; k += 2) ffma2(acc[r][k], acc[r][k + 1], wgt[r], f[k], f[k + 1]);
             }
         }
         __syncthreads();  // P, the scales and this stage's codes are free for the next chunk
