@@ -353,6 +353,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
         const int qw = warp - kEpiWarp0;         // job queue of this warp
         uint32_t* qjob = queue + qw * kQCap * 2;
         constexpr float qmaxf = (float)((1 << BITS) - 1);
+        constexpr float kRq = 1.0f / qmaxf;        // fl(1 / qmax)
+        constexpr float kBelow1 = 1.0f - 8.0f * kU;  // 1 - 2^-21 and 1 + 2^-21, both exact in fp32
+        constexpr float kAbove1 = 1.0f + 8.0f * kU;
         constexpr int qmax = (1 << BITS) - 1;
         constexpr int kJobSlots = NBK == 2 ? 4 : 2;  // values per lane and memory round trip
         int32_t flag = 0;
@@ -443,8 +446,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                 const float e = E[bk];
                 const float mn_lo = __fsub_rn(mn[bk], e), mn_hi = __fadd_rn(mn[bk], e);
                 const float mx_lo = __fsub_rn(mx[bk], e), mx_hi = __fadd_rn(mx[bk], e);
-                const uint32_t slo = f2h_bits(__fdiv_rn(fmaxf(__fsub_rn(mx_lo, mn_hi), 0.0f), qmaxf));
-                const uint32_t shi = scale16(mx_hi, mn_lo, qmaxf);
+                // fp16 scales of the smallest and largest possible ranges. fl(d * fl(1/qmax))
+                // is within (1 +- u)^2 of d / qmax and the widening product adds one more
+                // rounding, so the products widened by 8u bracket the IEEE quotients of both
+                // ends (which are within u of d / qmax); fp16 rounding is monotone, so equal
+                // roundings of the bracket decide the scale exactly (no division on this path)
+                const float dlo = fmaxf(__fsub_rn(mx_lo, mn_hi), 0.0f), dhi = __fsub_rn(mx_hi, mn_lo);
+                const uint32_t slo = f2h_bits(__fmul_rn(__fmul_rn(dlo, kRq), kBelow1));
+                const uint32_t shi = f2h_bits(__fmul_rn(__fmul_rn(dhi, kRq), kAbove1));
                 const uint32_t mlo = f2h_bits(mn_lo), mhi = f2h_bits(mn_hi);
                 s16[bk] = slo;
                 m16[bk] = mlo;
@@ -466,16 +475,33 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                     const bool nl = need != 0 && pickn(cmn, c) <= tl;
                     const bool nh = (need & 1) && pickn(cmx, c) >= th;
                     uint32_t m0 = 0, m1 = 0;
-                    if (__any_sync(0xffffffffu, nl || nh)) {
+                    const bool anyl = __any_sync(0xffffffffu, nl), anyh = __any_sync(0xffffffffu, nh);
+                    if (anyl || anyh) {
                         uint32_t v[32];
                         tmem_ld32(tacc + c * 32, v);
                         tmem_wait_ld();
+                        // sign bits of tl - z (z > tl) and z - th (z < th), one bit per column;
+                        // each side only when some lane of the warp needs it (with four blocks
+                        // per row, one loop for both keeps the row's state in registers)
                         uint32_t a0 = 0, a1 = 0;
+                        if constexpr (NBK == 4) {
 #pragma unroll
-                        for (int k = 31; k >= 0; k--) {
-                            const float z = __uint_as_float(v[k]);
-                            a0 = __funnelshift_l(__float_as_uint(__fsub_rn(tl, z)), a0, 1);
-                            a1 = __funnelshift_l(__float_as_uint(__fsub_rn(z, th)), a1, 1);
+                            for (int k = 31; k >= 0; k--) {
+                                const float z = __uint_as_float(v[k]);
+                                a0 = __funnelshift_l(__float_as_uint(__fsub_rn(tl, z)), a0, 1);
+                                a1 = __funnelshift_l(__float_as_uint(__fsub_rn(z, th)), a1, 1);
+                            }
+                        } else {
+                            if (anyl) {
+#pragma unroll
+                                for (int k = 31; k >= 0; k--)
+                                    a0 = __funnelshift_l(__float_as_uint(__fsub_rn(tl, __uint_as_float(v[k]))), a0, 1);
+                            }
+                            if (anyh) {
+#pragma unroll
+                                for (int k = 31; k >= 0; k--)
+                                    a1 = __funnelshift_l(__float_as_uint(__fsub_rn(__uint_as_float(v[k]), th)), a1, 1);
+                            }
                         }
                         m0 = nl ? ~a0 : 0u;  // z <= tl
                         m1 = nh ? ~a1 : 0u;  // z >= th
@@ -595,9 +621,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                 for (int w = 0; w < BITS; w++) words[w] = 0;
                 uint32_t mk = 0;
                 if (__all_sync(0xffffffffu, fst)) {
+                    // the same fma and add per value, two values per instruction
+                    const float2 r2 = make_float2(r, r), c2 = make_float2(cz, cz), m2 = make_float2(kMagic, kMagic);
 #pragma unroll
-                    for (int k = 0; k < 32; k++)
-                        put_code<BITS>(words, k, __float_as_uint(fmaf(__uint_as_float(v[k]), r, cz) + kMagic));
+                    for (int k = 0; k < 32; k += 2) {
+                        const float2 y = __fadd2_rn(
+                            __ffma2_rn(make_float2(__uint_as_float(v[k]), __uint_as_float(v[k + 1])), r2, c2), m2);
+                        put_code<BITS>(words, k, __float_as_uint(y.x));
+                        put_code<BITS>(words, k + 1, __float_as_uint(y.y));
+                    }
                 } else {
                     // clamping before the rounding gives the same code as clamping after it
                     const float lm = pickn(lim, bk);
