@@ -471,22 +471,25 @@ __global__ void __launch_bounds__(kThreads, 1) tc_decode_kernel(const __grid_con
                     ak[k] = m - kOff * s;
                 }
                 uint32_t o[16];
+                // the same multiply and fused multiply-adds per value, two columns per instruction
+                const float2 s0 = make_float2(sk[0], sk[0]), a0 = make_float2(ak[0], ak[0]);
+                const float2 s1 = make_float2(sk[1], sk[1]), a1 = make_float2(ak[1], ak[1]);
 #pragma unroll
                 for (int e = 0; e < 32; e += 4) {
                     const float4 c0 = *reinterpret_cast<const float4*>(cb + c * 32 + e);
-                    float x4[4] = {fmaf(sk[0], __uint_as_float(d0[e]), ak[0] * c0.x),
-                                   fmaf(sk[0], __uint_as_float(d0[e + 1]), ak[0] * c0.y),
-                                   fmaf(sk[0], __uint_as_float(d0[e + 2]), ak[0] * c0.z),
-                                   fmaf(sk[0], __uint_as_float(d0[e + 3]), ak[0] * c0.w)};
+                    float2 x01 = __ffma2_rn(s0, make_float2(__uint_as_float(d0[e]), __uint_as_float(d0[e + 1])),
+                                            __fmul2_rn(a0, make_float2(c0.x, c0.y)));
+                    float2 x23 = __ffma2_rn(s0, make_float2(__uint_as_float(d0[e + 2]), __uint_as_float(d0[e + 3])),
+                                            __fmul2_rn(a0, make_float2(c0.z, c0.w)));
                     if (nsub > 1) {
                         const float4 c1 = *reinterpret_cast<const float4*>(cb + kD + c * 32 + e);
-                        x4[0] = fmaf(sk[1], __uint_as_float(d1[e]), fmaf(ak[1], c1.x, x4[0]));
-                        x4[1] = fmaf(sk[1], __uint_as_float(d1[e + 1]), fmaf(ak[1], c1.y, x4[1]));
-                        x4[2] = fmaf(sk[1], __uint_as_float(d1[e + 2]), fmaf(ak[1], c1.z, x4[2]));
-                        x4[3] = fmaf(sk[1], __uint_as_float(d1[e + 3]), fmaf(ak[1], c1.w, x4[3]));
+                        x01 = __ffma2_rn(s1, make_float2(__uint_as_float(d1[e]), __uint_as_float(d1[e + 1])),
+                                         __ffma2_rn(a1, make_float2(c1.x, c1.y), x01));
+                        x23 = __ffma2_rn(s1, make_float2(__uint_as_float(d1[e + 2]), __uint_as_float(d1[e + 3])),
+                                         __ffma2_rn(a1, make_float2(c1.z, c1.w), x23));
                     }
-                    const __nv_bfloat162 b0 = __floats2bfloat162_rn(x4[0], x4[1]);
-                    const __nv_bfloat162 b1 = __floats2bfloat162_rn(x4[2], x4[3]);
+                    const __nv_bfloat162 b0 = __floats2bfloat162_rn(x01.x, x01.y);
+                    const __nv_bfloat162 b1 = __floats2bfloat162_rn(x23.x, x23.y);
                     o[e >> 1] = *reinterpret_cast<const uint32_t*>(&b0);
                     o[(e >> 1) + 1] = *reinterpret_cast<const uint32_t*>(&b1);
                 }

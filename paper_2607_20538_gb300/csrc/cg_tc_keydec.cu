@@ -287,18 +287,24 @@ __global__ void __launch_bounds__(kThreads, 1) tc_key_decode_kernel(const KdPara
                 uint32_t hi[4], lo[4];
 #pragma unroll
                 for (int e = 0; e < 4; e++) {
-                    float z2[2];
+                    // q as fp32 without an integer conversion: 2^23 + q has q in its low
+                    // mantissa bits, and subtracting 2^23 is exact
+                    uint32_t qb[2];
 #pragma unroll
                     for (int u = 0; u < 2; u++) {
                         const int t = 8 * c + 2 * e + u;
                         const int p = t * BITS;
                         uint32_t v = w[p >> 5] >> (p & 31);
                         if ((p & 31) + BITS > 32) v |= w[(p >> 5) + 1] << (32 - (p & 31));
-                        z2[u] = fmaf((float)(v & ((1u << BITS) - 1u)), s, m);
+                        qb[u] = (v & ((1u << BITS) - 1u)) | 0x4B000000u;
                     }
-                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(z2[0], z2[1]);
+                    const float2 qf = __fadd2_rn(make_float2(__uint_as_float(qb[0]), __uint_as_float(qb[1])),
+                                                 make_float2(-8388608.0f, -8388608.0f));
+                    const float2 z2 = __ffma2_rn(qf, make_float2(s, s), make_float2(m, m));  // q s + m
+                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(z2.x, z2.y);
                     const float2 hf = __bfloat1622float2(h2);
-                    const __nv_bfloat162 l2 = __floats2bfloat162_rn(z2[0] - hf.x, z2[1] - hf.y);
+                    const float2 r2 = __fadd2_rn(z2, make_float2(-hf.x, -hf.y));  // exact
+                    const __nv_bfloat162 l2 = __floats2bfloat162_rn(r2.x, r2.y);
                     hi[e] = *reinterpret_cast<const uint32_t*>(&h2);
                     lo[e] = *reinterpret_cast<const uint32_t*>(&l2);
                 }
