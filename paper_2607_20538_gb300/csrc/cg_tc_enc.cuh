@@ -83,7 +83,7 @@ __device__ __forceinline__ void run_jobs(uint32_t* qjob, int nq, const unsigned 
             const int kk = (col & ~(g - 1)) + 4 * j;  // first channel of this lane's products
             xv[k] = *reinterpret_cast<const uint2*>(stage + (kk >> 6) * 16384 + row * 128 +
                                                     ((((kk & 63) >> 3) ^ (row & 7)) << 4) + (kk & 7) * 2);
-            gv[k] = __ldg(reinterpret_cast<const float4*>(Gf + (size_t)col * g + 4 * j));
+            gv[k] = ldg_hint_f4(Gf + (size_t)col * g + 4 * j, policy_evict_last());  // kept in L2
         }
         float part[kSlots];
 #pragma unroll
@@ -148,7 +148,7 @@ __device__ __forceinline__ void prefetch_next_gauges(const RowArgs& a, const tc:
     }
     if (nl < a.L) {
         const char* nG = reinterpret_cast<const char*>(a.G + ((int64_t)(nl * 2 + ns) * a.H + nh) * (int64_t)kD * g);
-        for (int off = lane * 128; off < kD * g * 4; off += 32 * 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(nG + off));
+        for (int off = lane * 128; off < kD * g * 4; off += 32 * 128) asm volatile("prefetch.global.L2::evict_last [%0];" ::"l"(nG + off));
     }
 }
 

@@ -247,8 +247,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                 const int64_t row0 = tc::dense_row(a, ti);
                 unsigned char* dst = stages + st * kTileBytes;
                 mbar_arrive_expect_tx(&M->full[st], kTileBytes);
-                tma_load_2d(dst, &xmap, &M->full[st], 0, (int)row0);
-                tma_load_2d(dst + 16384, &xmap, &M->full[st], 64, (int)row0);
+                // the cache tiles are read once: first out of L2, so that the gauge sets the
+                // exact recomputes read stay there
+                const uint64_t pol = policy_evict_first();
+                tma_load_2d_hint(dst, &xmap, &M->full[st], 0, (int)row0, pol);
+                tma_load_2d_hint(dst + 16384, &xmap, &M->full[st], 64, (int)row0, pol);
                 issued = i + 1;
             }
             if (*abort_flag) {
@@ -649,8 +652,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_rows_encode_kernel(const __gri
                     uint32_t* dst = reinterpret_cast<uint32_t*>(crow) + c * BITS;
                     if constexpr (BITS % 4 == 0) {
 #pragma unroll
-                        for (int w = 0; w < BITS; w += 4)
-                            *reinterpret_cast<uint4*>(dst + w) = make_uint4(words[w], words[w + 1], words[w + 2], words[w + 3]);
+                        for (int w = 0; w < BITS; w += 4)  // written once: first out of L2
+                            stg_hint_u4(dst + w, make_uint4(words[w], words[w + 1], words[w + 2], words[w + 3]),
+                                        policy_evict_first());
                     } else if constexpr (BITS % 2 == 0) {
 #pragma unroll
                         for (int w = 0; w < BITS; w += 2) *reinterpret_cast<uint2*>(dst + w) = make_uint2(words[w], words[w + 1]);
